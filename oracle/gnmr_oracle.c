@@ -1,0 +1,301 @@
+/*
+ * GNMR oracle: a plain, slow, double-precision CPU restatement of the GNMR
+ * per-step monitor (GNMR: Runtime Stability Control for Low-Precision LLM
+ * Training).
+ *
+ * TEST INFRASTRUCTURE ONLY.  The tests, the smoke check and the benchmark's
+ * CPU baseline may load this file's library; the product (the CUDA path in
+ * the package) never does, and shares no code, header or table with it.
+ *
+ * What it computes, in the paper's order and notation:
+ *   - n_{b,t} = ||g_{b,t}||_2 for every monitored unit b      (Sec. 2, Eq. local_gradient)
+ *   - Algorithm 1: GNMR_{b,t}, Delta-GNMR_{b,t}, A_{b,t}, Q_b   (Sec. 3.1-3.2, Alg. 1)
+ *   - Algorithm 2: R_{b,t}, C_t, A_t = Top_maxO(C_t; R), Lock_b (Sec. 3.3, Alg. 2)
+ *
+ * Readings taken where the paper is silent (each one is listed with its
+ * reason in the design notes):
+ *   - "t = 1" in Algorithm 1 is read per unit: k_b, the number of steps at
+ *     which unit b was observed, plays the role of t (equal to the global t
+ *     whenever every step is observed).
+ *   - A non-finite norm (NaN or Inf) gives GNMR = Delta-GNMR = R = +Inf and
+ *     leaves A_b, Q_b and k_b untouched.
+ *   - mean(Q_b) + eps == 0 gives Delta-GNMR = +Inf if GNMR > 0, else 1.
+ *   - Top_maxO orders by R descending, then by unit index ascending, and
+ *     selects min(maxO, |C_t|) units.
+ *   - alpha_t, beta_t: the *_init values for t <= warmup_steps, the *_main
+ *     values after, unless the caller overrides them for the step.
+ *
+ * Build: gcc -O2 -shared -fPIC -o liboracle_gnmr.so gnmr_oracle.c -lm
+ * (no fast-math: every sum below runs in the order written).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_DTYPE_F32 0
+#define ORACLE_DTYPE_BF16 1
+
+/* A bfloat16 value is the upper 16 bits of an IEEE-754 binary32 value, so
+ * shifting it into place gives the exact binary32 (and then binary64) value. */
+static double bf16_to_double(uint16_t h)
+{
+    uint32_t bits = ((uint32_t)h) << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+/* Eq. local_gradient: n_b = ||g_b||_2, the square root of the sum of squares
+ * of every element of unit b's segment, summed sequentially in double. */
+int oracle_unit_norms(const void *arena, int dtype, const int64_t *offsets,
+                      const int64_t *lengths, int32_t num_units, double *norms)
+{
+    if (dtype != ORACLE_DTYPE_F32 && dtype != ORACLE_DTYPE_BF16)
+        return 1;
+    for (int32_t b = 0; b < num_units; ++b) {
+        double sum = 0.0;
+        if (dtype == ORACLE_DTYPE_F32) {
+            const float *g = (const float *)arena + offsets[b];
+            for (int64_t i = 0; i < lengths[b]; ++i) {
+                double x = (double)g[i];
+                sum += x * x;
+            }
+        } else {
+            const uint16_t *g = (const uint16_t *)arena + offsets[b];
+            for (int64_t i = 0; i < lengths[b]; ++i) {
+                double x = bf16_to_double(g[i]);
+                sum += x * x;
+            }
+        }
+        norms[b] = sqrt(sum);
+    }
+    return 0;
+}
+
+/* Per-unit controller state: A_b (historical mean), Q_b (the last <= delta
+ * GNMR values, oldest first), k_b (observation count), Lock_b. */
+typedef struct {
+    int32_t num_units;
+    int32_t window;      /* delta */
+    int32_t max_o;       /* maxO */
+    int32_t lock_len;    /* T_lock */
+    int64_t warmup_steps;
+    double alpha_init, alpha_main, beta_init, beta_main, eps;
+    int64_t t;           /* completed steps */
+    uint8_t *recoverable;
+    double *A;
+    int64_t *k;
+    double *Q;           /* num_units * window, oldest first */
+    int32_t *qlen;
+    int32_t *lock;
+    int32_t *cand;       /* scratch for Algorithm 2 */
+} oracle_ctl;
+
+void oracle_ctl_destroy(oracle_ctl *c)
+{
+    if (!c)
+        return;
+    free(c->recoverable);
+    free(c->A);
+    free(c->k);
+    free(c->Q);
+    free(c->qlen);
+    free(c->lock);
+    free(c->cand);
+    free(c);
+}
+
+oracle_ctl *oracle_ctl_create(int32_t num_units, int32_t window, int32_t max_o,
+                              int32_t lock_len, int64_t warmup_steps,
+                              double alpha_init, double alpha_main,
+                              double beta_init, double beta_main, double eps,
+                              const uint8_t *recoverable)
+{
+    if (num_units < 1 || window < 1 || max_o < 0 || lock_len < 0)
+        return NULL;
+    oracle_ctl *c = (oracle_ctl *)calloc(1, sizeof *c);
+    if (!c)
+        return NULL;
+    c->num_units = num_units;
+    c->window = window;
+    c->max_o = max_o;
+    c->lock_len = lock_len;
+    c->warmup_steps = warmup_steps;
+    c->alpha_init = alpha_init;
+    c->alpha_main = alpha_main;
+    c->beta_init = beta_init;
+    c->beta_main = beta_main;
+    c->eps = eps;
+    size_t u = (size_t)num_units;
+    c->recoverable = (uint8_t *)calloc(u, 1);
+    c->A = (double *)calloc(u, sizeof(double));
+    c->k = (int64_t *)calloc(u, sizeof(int64_t));
+    c->Q = (double *)calloc(u * (size_t)window, sizeof(double));
+    c->qlen = (int32_t *)calloc(u, sizeof(int32_t));
+    c->lock = (int32_t *)calloc(u, sizeof(int32_t));
+    c->cand = (int32_t *)calloc(u, sizeof(int32_t));
+    if (!c->recoverable || !c->A || !c->k || !c->Q || !c->qlen || !c->lock || !c->cand) {
+        oracle_ctl_destroy(c);
+        return NULL;
+    }
+    for (size_t b = 0; b < u; ++b)
+        c->recoverable[b] = recoverable ? (recoverable[b] != 0) : 1;
+    return c;
+}
+
+/* Algorithm 1 for one unit: returns GNMR and Delta-GNMR through g and d, and
+ * updates A_b, k_b and Q_b. */
+static void algorithm1(oracle_ctl *c, int32_t b, double n, double *g, double *d)
+{
+    double *Qb = c->Q + (size_t)b * (size_t)c->window;
+    double gnmr, dgnmr;
+
+    if (!isfinite(n)) {           /* reading: non-finite norm, no state update */
+        *g = INFINITY;
+        *d = INFINITY;
+        return;
+    }
+    /* GNMR: 1 at the unit's first step or while the historical mean is 0. */
+    if (c->k[b] == 0 || c->A[b] == 0.0)
+        gnmr = 1.0;
+    else
+        gnmr = n / (c->A[b] + c->eps);
+
+    /* Delta-GNMR: GNMR over the mean of the last delta GNMR values, once the
+     * queue holds delta values; 1 before that. */
+    if (c->qlen[b] == c->window) {
+        double s = 0.0;
+        for (int32_t i = 0; i < c->window; ++i)
+            s += Qb[i];
+        double denom = s / (double)c->window + c->eps;
+        if (denom == 0.0)
+            dgnmr = (gnmr > 0.0) ? INFINITY : 1.0;
+        else
+            dgnmr = gnmr / denom;
+    } else {
+        dgnmr = 1.0;
+    }
+
+    /* Incremental mean A_{b,t} = A_{b,t-1} + (n - A_{b,t-1}) / t. */
+    c->k[b] += 1;
+    c->A[b] = c->A[b] + (n - c->A[b]) / (double)c->k[b];
+
+    /* Push GNMR into Q_b, keeping only the most recent delta values. */
+    if (c->qlen[b] == c->window) {
+        for (int32_t i = 0; i + 1 < c->window; ++i)
+            Qb[i] = Qb[i + 1];
+        Qb[c->window - 1] = gnmr;
+    } else {
+        Qb[c->qlen[b]] = gnmr;
+        c->qlen[b] += 1;
+    }
+    *g = gnmr;
+    *d = dgnmr;
+}
+
+/* qsort has no user pointer: the comparator reads R through this
+ * thread-local variable. */
+static _Thread_local const double *g_sort_r;
+
+static int by_risk_then_index(const void *pa, const void *pb)
+{
+    int32_t a = *(const int32_t *)pa, b = *(const int32_t *)pb;
+    double ra = g_sort_r[a], rb = g_sort_r[b];
+    if (ra > rb)
+        return -1;
+    if (ra < rb)
+        return 1;
+    return (a < b) ? -1 : (a > b);
+}
+
+/* One training step: Algorithm 1 for every monitored unit, then Algorithm 2.
+ * alpha_override / beta_override: NaN selects the two-stage schedule.
+ * Outputs (each num_units long): gnmr, dgnmr, risk, mask (1 = recovery
+ * path), lock_out (Lock_b after the step).  counts[0] = |C_t|,
+ * counts[1] = |A_t|. */
+int oracle_ctl_step(oracle_ctl *c, const double *norms, double alpha_override,
+                    double beta_override, double *gnmr, double *dgnmr,
+                    double *risk, uint8_t *mask, int32_t *lock_out,
+                    int32_t *counts)
+{
+    int32_t U = c->num_units;
+
+    for (int32_t b = 0; b < U; ++b)
+        algorithm1(c, b, norms[b], &gnmr[b], &dgnmr[b]);
+
+    c->t += 1;
+    double alpha = isnan(alpha_override)
+                       ? (c->t <= c->warmup_steps ? c->alpha_init : c->alpha_main)
+                       : alpha_override;
+    double beta = isnan(beta_override)
+                      ? (c->t <= c->warmup_steps ? c->beta_init : c->beta_main)
+                      : beta_override;
+
+    /* R_{b,t} = max{GNMR / alpha_t, Delta-GNMR / beta_t}. */
+    for (int32_t b = 0; b < U; ++b) {
+        double x = gnmr[b] / alpha, y = dgnmr[b] / beta;
+        risk[b] = (x > y) ? x : y;
+    }
+
+    /* C_t = {b : R > 1} U {b : Lock_b > 0}, over recoverable units only. */
+    int32_t ncand = 0;
+    for (int32_t b = 0; b < U; ++b)
+        if (c->recoverable[b] && (risk[b] > 1.0 || c->lock[b] > 0))
+            c->cand[ncand++] = b;
+
+    /* A_t = Top_maxO(C_t; R): sort by R descending, index ascending. */
+    g_sort_r = risk;
+    qsort(c->cand, (size_t)ncand, sizeof(int32_t), by_risk_then_index);
+    int32_t nsel = ncand < c->max_o ? ncand : c->max_o;
+
+    for (int32_t b = 0; b < U; ++b)
+        mask[b] = 0;
+    for (int32_t i = 0; i < nsel; ++i)
+        mask[c->cand[i]] = 1;
+
+    /* Lock bookkeeping of Algorithm 2. */
+    for (int32_t b = 0; b < U; ++b) {
+        if (!c->recoverable[b]) {
+            c->lock[b] = 0;
+        } else if (mask[b]) {
+            if (risk[b] > 1.0)
+                c->lock[b] = c->lock_len;
+            else
+                c->lock[b] = (c->lock[b] - 1 > 0) ? c->lock[b] - 1 : 0;
+        } else {
+            c->lock[b] = 0;
+        }
+        lock_out[b] = c->lock[b];
+    }
+    counts[0] = ncand;
+    counts[1] = nsel;
+    return 0;
+}
+
+/* State access, for checkpoint/resume tests: A[U], k[U], Q[U*window] (oldest
+ * first, qlen[b] valid entries), qlen[U], lock[U], t. */
+void oracle_ctl_get_state(const oracle_ctl *c, double *A, int64_t *k, double *Q,
+                          int32_t *qlen, int32_t *lock, int64_t *t)
+{
+    size_t u = (size_t)c->num_units;
+    memcpy(A, c->A, u * sizeof(double));
+    memcpy(k, c->k, u * sizeof(int64_t));
+    memcpy(Q, c->Q, u * (size_t)c->window * sizeof(double));
+    memcpy(qlen, c->qlen, u * sizeof(int32_t));
+    memcpy(lock, c->lock, u * sizeof(int32_t));
+    *t = c->t;
+}
+
+void oracle_ctl_set_state(oracle_ctl *c, const double *A, const int64_t *k,
+                          const double *Q, const int32_t *qlen,
+                          const int32_t *lock, int64_t t)
+{
+    size_t u = (size_t)c->num_units;
+    memcpy(c->A, A, u * sizeof(double));
+    memcpy(c->k, k, u * sizeof(int64_t));
+    memcpy(c->Q, Q, u * (size_t)c->window * sizeof(double));
+    memcpy(c->qlen, qlen, u * sizeof(int32_t));
+    memcpy(c->lock, lock, u * sizeof(int32_t));
+    c->t = t;
+}
