@@ -1,0 +1,409 @@
+#!/usr/bin/env python
+"""Benchmark of the GNMR per-step monitor on GB300.
+
+One step = one gnmr_step over one full synthetic gradient arena: every unit's
+L2 norm, Algorithm 1, the combined risk, Top_maxO with the lock bookkeeping
+and the mask write (one kernel launch).  The default workload is the
+LLaMA-2-13B layout: 40 layers x 7 linears = 280 bf16 units, 12.69 G elements
+(25.38 GB) per step, larger than L2, so no flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gnmr|reference]
+
+Prints one JSON line (rank 0).  Under torchrun (N > 1) each rank runs an
+independent replica on its own GPU (the monitor has no exchange step on one
+replica); time is the max over ranks and `value` counts every rank's bytes.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "GNMR step µs & grad GB/s (% HBM peak), LLaMA-2-13B 280-unit layout"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args(argv=None):
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["gnmr", "reference"], default="gnmr")
+    p.add_argument("--workload", default="llama2-13b")
+    p.add_argument("--shrink", type=int, default=1,
+                   help="divide matrix dims (small case for profiler captures)")
+    p.add_argument("--arenas", type=int, default=2, help="distinct step arenas cycled")
+    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-sample-units", type=int, default=0,
+                   help="units in the CPU-oracle sample (0 = all: one full step)")
+    p.add_argument("--ref-sample-units", type=int, default=42,
+                   help="units per step of the reference arm (host-generated)")
+    return p.parse_args(argv)
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (replicas only)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Max of a per-rank float over all ranks (identity for one rank)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int, device=None):
+    if world > 1:
+        import torch.distributed as dist
+        if device is not None and dist.get_backend() == "nccl":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, interval_ms: int = 20):
+        self.rows = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(gpu_index), "-lms", str(interval_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=5)
+
+    def summary(self, t0: float, t1: float) -> dict:
+        inside = [r for ts, r in self.rows if t0 <= ts <= t1]
+        window = "timed region"
+        if not inside:
+            inside = [r for ts, r in self.rows if t0 - 0.5 <= ts <= t1 + 0.5]
+            window = "within 0.5 s of the timed region"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "note": "nvidia-smi gave no sample"}
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[2]) for r in inside if num(r[2]) is not None]
+        mx = [num(r[3]) for r in inside if num(r[3]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i in range(4)
+                          if len(r) > 6 + i and r[6 + i].lower().startswith("active")})
+        power = [num(r[4]) for r in inside if num(r[4]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(inside), "window": window,
+                "power_w_max": max(power) if power else None}
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the oracle on a bounded sample of the same workload
+# ---------------------------------------------------------------------------
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_oracle_rate(view, w, units, reps: int = 1):
+    """Times the oracle (norms of `units` + Algorithms 1-2 over them) and
+    returns (GB/s, threads, seconds per rep)."""
+    import oracle
+    off = w.offsets[units]
+    ln = w.lengths[units]
+    threads = min(host_cores(), len(units))
+    ctl = oracle.Controller(len(units), **dict(w.controller_kwargs(),
+                                               recoverable=w.recoverable[units]))
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        n = oracle.unit_norms_threaded(view, off, ln, threads)
+        ctl.step(n)
+        times.append(time.perf_counter() - t0)
+    ctl.close()
+    sec = statistics.median(times)
+    nbytes = int(ln.sum()) * w.elem_bytes
+    return nbytes / sec / 1e9, threads, sec
+
+
+def bf16_bits(x: np.ndarray) -> np.ndarray:
+    """float32 -> bfloat16 bit patterns, round to nearest even."""
+    u = x.astype(np.float32).view(np.uint32)
+    r = ((u >> 16) & 1) + 0x7FFF
+    return ((u + r) >> 16).astype(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the oracle on the host cores
+# ---------------------------------------------------------------------------
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    import workloads
+    w = workloads.make(args.workload, shrink=args.shrink)
+    units = np.arange(min(args.ref_sample_units, w.num_units))
+    off = w.offsets[units]
+    ln = w.lengths[units]
+    rng = np.random.default_rng(0)
+    # host-generated sample arena (same unit sizes and scale model)
+    local_off = np.concatenate([[0], np.cumsum(ln)[:-1]]).astype(np.int64)
+    arena = np.empty(int(ln.sum()), dtype=np.uint16 if w.dtype == "bf16" else np.float32)
+    for i, u in enumerate(units):
+        z = (rng.standard_normal(int(ln[i])) * w.scales[0, u]).astype(np.float32)
+        arena[local_off[i]:local_off[i] + ln[i]] = bf16_bits(z) if w.dtype == "bf16" else z
+    threads = min(host_cores(), len(units))
+    ctl = oracle.Controller(len(units), **dict(w.controller_kwargs(),
+                                               recoverable=w.recoverable[units]))
+    for _ in range(args.warmup):
+        ctl.step(oracle.unit_norms_threaded(arena, local_off, ln, threads))
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ctl.step(oracle.unit_norms_threaded(arena, local_off, ln, threads))
+    sec = (time.perf_counter() - t0) / max(args.steps, 1)
+    ctl.close()
+    nbytes = int(ln.sum()) * w.elem_bytes
+    gbs = nbytes / sec / 1e9
+    sample = (f"units 0..{len(units) - 1} of the {w.num_units}-unit {w.name} layout "
+              f"({nbytes / 1e9:.3f} GB of {w.grad_bytes / 1e9:.3f} GB per step), host-generated")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(gbs, 4), "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(w.grad_bytes / (gbs * 1e9) * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+        "data": "synthetic",
+        "config": {"workload": f"{w.name} ({w.num_units} units, {w.grad_elems} {w.dtype} elements)",
+                   "bytes_per_step": w.grad_bytes},
+        "cpu_baseline": {"value": round(gbs, 4), "unit": "GB/s", "cores": threads,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(gbs, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "note": "ms_per_step extrapolates the sample rate to the full step",
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+def run_gnmr(args):
+    import torch
+    import workloads
+    from paper_2606_00539_gb300 import Monitor
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+
+    w = workloads.make(args.workload, shrink=args.shrink, seed=rank)
+    filler = workloads.Filler(w, dev)
+    n_arenas = max(1, args.arenas)
+    arenas = []
+    for i in range(n_arenas):
+        a = filler.new_arena()
+        filler.fill(a, i % w.steps)
+        arenas.append(a)
+    mon = Monitor(w.offsets, w.lengths, device=local_rank, **w.monitor_kwargs())
+    info = mon.info()
+    stats = mon.new_stats()
+    mask = torch.empty(w.num_units, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(dev)
+    torch.cuda.synchronize(dev)
+
+    for i in range(args.warmup):
+        mon.step(arenas[i % n_arenas], mask=mask, stats=stats, stream=stream)
+    stream.synchronize()
+
+    sampler = ClockSampler(local_rank)
+    time.sleep(0.3)                       # let nvidia-smi start sampling
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    barrier(world, dev)
+    torch.cuda.synchronize(dev)
+    wall0 = time.time()
+    t_start.record(stream)
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        mon.step(arenas[(args.warmup + i) % n_arenas], mask=mask, stats=stats, stream=stream)
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    stream.synchronize()
+    torch.cuda.synchronize(dev)
+    wall1 = time.time()
+    barrier(world, dev)
+    sampler.stop()
+    clocks = sampler.summary(wall0, wall1)
+
+    total_ms = t_start.elapsed_time(t_end)
+    per_ms = [a.elapsed_time(b) for a, b in ev]
+    max_ms = max_over_ranks(total_ms, world, dev)
+    launches = args.steps                              # one kernel per gnmr_step
+
+    gbytes = w.grad_bytes / 1e9
+    value = world * gbytes * args.steps / (max_ms / 1e3)
+    step_ms = max_ms / args.steps
+    kern_ms = statistics.mean(per_ms)
+    peak, peak_kind = measured_peaks()
+    achieved = gbytes / (kern_ms / 1e3)
+
+    # end to end through the public API: host arena (pinned) -> device, the
+    # step, the mask back to the host, every step inside the timed region
+    e2e = None
+    host = None
+    if not args.no_e2e and args.e2e_steps > 0:
+        try:
+            host = torch.empty(arenas[0].numel(), dtype=arenas[0].dtype, pin_memory=True)
+            host.copy_(arenas[0])
+            host_mask = torch.empty(w.num_units, dtype=torch.uint8, pin_memory=True)
+            dst = arenas[-1]
+            for i in range(args.e2e_steps + 1):
+                if i == 1:
+                    torch.cuda.synchronize(dev)
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                with torch.cuda.stream(stream):
+                    dst.copy_(host, non_blocking=True)
+                    mon.step(dst, mask=mask, stream=stream)
+                    host_mask.copy_(mask, non_blocking=True)
+                stream.synchronize()
+            e1.record(stream)
+            stream.synchronize()
+            e2e_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
+            e2e = {"value": round(world * gbytes / (e2e_ms / 1e3), 3), "unit": "GB/s",
+                   "ms_per_step": round(e2e_ms, 3),
+                   "h2d_bytes_per_step": int(host.numel() * host.element_size()),
+                   "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
+                   "path": "pinned host arena -> device copy, gnmr_step, mask -> pinned host"}
+        except RuntimeError as exc:
+            e2e = {"value": None, "unit": "GB/s", "error": str(exc).splitlines()[0]}
+            host = None
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        k = args.cpu_sample_units or w.num_units
+        units = np.arange(min(k, w.num_units))
+        hi = int(w.offsets[units[-1]] + w.lengths[units[-1]])
+        src = host[:hi] if host is not None else arenas[0][:hi].cpu()
+        view = src.view(torch.int16).numpy().view(np.uint16) if w.dtype == "bf16" else src.numpy()
+        rate, threads, sec = cpu_oracle_rate(view, w, units)
+        what = ("one full step" if len(units) == w.num_units
+                else f"units 0..{len(units) - 1} of {w.num_units}")
+        cpu = {"value": round(rate, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+               "sample": (f"{what} ({int(w.lengths[units].sum()) * w.elem_bytes / 1e9:.3f} GB of "
+                          f"{gbytes:.3f} GB per step): unit norms + Algorithms 1-2, "
+                          f"{sec:.2f} s wall on {threads} threads")}
+    del host
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_ms, 4),
+            "us_per_step": round(step_ms * 1e3, 1),
+            "pct_hbm_peak": round(100 * value / world / peak, 2),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": f"{w.name} ({w.num_units} units, {w.grad_elems} {w.dtype} "
+                                   f"elements{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
+                       "bytes_per_step": w.grad_bytes, "arenas_cycled": n_arenas,
+                       "l2": "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * 129e6
+                       else "inputs fit in L2 (hot)",
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
+                               f"{info['num_warps']} warp runs"},
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                         "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                         "peak_source": f"{peak_kind} hbm_gbs", "kernel": "gnmr_step_kernel<bf16>",
+                         "kernel_ms_mean": round(kern_ms, 4),
+                         "kernel_ms_min": round(min(per_ms), 4)},
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    mon.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gnmr(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,184 @@
+/*
+ * gnmr.h -- C ABI of libgnmr, the GB300 (sm_103a) implementation of the GNMR
+ * per-step monitor: per-unit gradient L2 norms, the online GNMR and
+ * Delta-GNMR statistics, and the budgeted choice of the units that move to
+ * the higher-fidelity recovery path.
+ *
+ * Paper: "GNMR: Runtime Stability Control for Low-Precision Large Language
+ * Model Training".  Definitions implemented here:
+ *   Sec. 2, Eq. local_gradient   n_{b,t} = ||g_{b,t}||_2 per monitored unit b
+ *   Sec. 3.1-3.2, Algorithm 1    GNMR, Delta-GNMR, historical mean A, queue Q
+ *   Sec. 3.3, Algorithm 2        R = max{GNMR/alpha_t, Delta-GNMR/beta_t},
+ *                                C_t = {R > 1} U {Lock > 0}, A_t = Top_maxO,
+ *                                Lock bookkeeping
+ *   Sec. 3.4                     recoverable vs monitored units, maxO as a
+ *                                hard cap, two-stage thresholds
+ *
+ * Conventions shared by every call:
+ *   - Every call returns a gnmr_status; GNMR_OK is 0.  A call that fails its
+ *     argument or layout checks returns before anything is enqueued and
+ *     leaves the handle's state (step counter included) unchanged.
+ *   - Pointers named d_* are CUDA device pointers on the handle's device;
+ *     every other pointer is host memory.
+ *   - The library owns its state and scratch: one device allocation made by
+ *     gnmr_create and freed by gnmr_destroy.  The caller owns the gradient
+ *     arena, the mask and the statistics buffers.
+ *   - Work is enqueued on the caller's stream (a cudaStream_t passed as
+ *     void*, NULL = the legacy default stream).  gnmr_step never blocks the
+ *     host; its outputs are valid once that stream reaches the step.
+ *   - A handle is not thread-safe: one host thread and one stream at a time.
+ *   - The calls save and restore the caller's current CUDA device.
+ */
+#ifndef GNMR_H
+#define GNMR_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum gnmr_status {
+    GNMR_OK = 0,
+    GNMR_ERR_INVALID_ARG = 1, /* bad pointer, size, threshold or config value */
+    GNMR_ERR_LAYOUT = 2,      /* unit layout does not fit the arena given */
+    GNMR_ERR_CUDA = 3,        /* a CUDA call failed; the handle is then only good for destroy */
+    GNMR_ERR_OOM = 4,         /* host or device allocation failed in gnmr_create */
+    GNMR_ERR_STATE = 5        /* handle unusable after an earlier GNMR_ERR_CUDA */
+} gnmr_status;
+
+typedef enum gnmr_dtype {
+    GNMR_DTYPE_F32 = 0,       /* IEEE binary32 gradients */
+    GNMR_DTYPE_BF16 = 1       /* bfloat16 gradients */
+} gnmr_dtype;
+
+/* Controller configuration (Sec. 3.3-3.4).  gnmr_config_defaults fills it
+ * with the values listed per field. */
+typedef struct gnmr_config {
+    int32_t num_units;            /* |B|, monitored units, >= 1 (no default) */
+    const int64_t *offsets;       /* host [num_units]: first element of unit b in the arena, >= 0 */
+    const int64_t *lengths;       /* host [num_units]: elements of unit b, >= 0 (0 = empty unit, norm 0) */
+    const uint8_t *recoverable;   /* host [num_units], nonzero = b in B_rec; NULL = every unit recoverable */
+    int32_t dtype;                /* gnmr_dtype of the arena; default GNMR_DTYPE_BF16 */
+    int32_t window;               /* delta, Delta-GNMR window, >= 1; default 8 */
+    int32_t max_o;                /* maxO, hard cap on |A_t|, >= 0; default 4 */
+    int32_t lock_len;             /* T_lock, >= 0; default 1 */
+    double alpha_init;            /* alpha_t for t <= warmup_steps, > 0; default 1.5 */
+    double alpha_main;            /* alpha_t for t > warmup_steps, > 0; default 1.1 */
+    double beta_init;             /* beta_t for t <= warmup_steps, > 0; default 1.5 */
+    double beta_main;             /* beta_t for t > warmup_steps, > 0; default 1.5 */
+    int64_t warmup_steps;         /* length of the first threshold stage, >= 0; default 0 */
+    double eps;                   /* epsilon of Algorithm 1, >= 0; default 1e-8 */
+    int32_t device;               /* CUDA device ordinal; default 0 */
+} gnmr_config;
+
+/* Optional per-step statistics: caller-owned DEVICE buffers.  Any pointer
+ * may be NULL, and the whole struct may be NULL. */
+typedef struct gnmr_stats {
+    double *norm;     /* [num_units] n_{b,t} */
+    double *gnmr;     /* [num_units] GNMR_{b,t} */
+    double *dgnmr;    /* [num_units] Delta-GNMR_{b,t} */
+    double *risk;     /* [num_units] R_{b,t} (also reported for non-recoverable units) */
+    int32_t *lock;    /* [num_units] Lock_b after the step */
+    int32_t *counts;  /* [2]: |C_t|, |A_t| */
+} gnmr_stats;
+
+/* Launch geometry and memory of a handle, for reporting. */
+typedef struct gnmr_info {
+    int32_t num_units;
+    int32_t dtype;
+    int32_t device;
+    int32_t num_ctas;          /* CTAs per gnmr_step launch */
+    int32_t threads_per_cta;
+    int32_t num_warps;         /* warps with a non-empty work run */
+    int64_t num_partials;      /* per-(warp, unit) partial sums */
+    int64_t device_bytes;      /* library-owned device memory */
+    int64_t arena_elems_min;   /* max over units of offset + length */
+    int64_t steps;             /* gnmr_step calls enqueued so far */
+} gnmr_info;
+
+typedef struct gnmr_handle gnmr_handle;
+
+/* Fills *cfg with the defaults documented in gnmr_config; num_units,
+ * offsets, lengths and recoverable are set to 0 / NULL.  cfg may not be NULL
+ * (the call then does nothing). */
+void gnmr_config_defaults(gnmr_config *cfg);
+
+/* Validates cfg, copies the unit layout and recoverable flags (the caller may
+ * free them afterwards), plans the work partition for the device, allocates
+ * and zeroes the per-unit state (A_b, Q_b, k_b, Lock_b) and scratch, and
+ * returns a handle in *out.  This is the only call that allocates or blocks.
+ * Errors: GNMR_ERR_INVALID_ARG (NULL cfg/out/offsets/lengths, a field out of
+ * range, offset + length overflowing), GNMR_ERR_CUDA (device not usable),
+ * GNMR_ERR_OOM.  On error *out is set to NULL; gnmr_last_error(NULL) gives
+ * the detail. */
+gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out);
+
+/* One training step t = (steps so far) + 1, one kernel launch on `stream`:
+ *   1. n_b = ||g_b||_2 for every unit b over the arena (Eq. local_gradient);
+ *   2. Algorithm 1 for every unit (k_b plays the role of t: the number of
+ *      steps at which b was observed);
+ *   3. R_b = max{GNMR/alpha_t, Delta-GNMR/beta_t} (Sec. 3.3), with alpha_t,
+ *      beta_t from the two-stage schedule or gnmr_set_thresholds;
+ *   4. C_t = {b in B_rec : R_b > 1 or Lock_b > 0};
+ *      A_t = the min(maxO, |C_t|) members of C_t with the largest R, ties
+ *      broken by the lower unit index (Algorithm 2);
+ *   5. Lock_b = T_lock if b in A_t and R_b > 1; max(Lock_b - 1, 0) if b in
+ *      A_t and R_b <= 1; 0 otherwise; d_mask[b] = 1 iff b in A_t.
+ * A unit whose norm is NaN or Inf gets GNMR = Delta-GNMR = R = +Inf and its
+ * A_b, Q_b and k_b are left as they were.
+ * Arguments:
+ *   d_arena      device, the flat gradient arena of the configured dtype,
+ *                aligned to its element size; read only.  May be NULL only
+ *                if every unit is empty.
+ *   arena_elems  elements in d_arena; must be >= max(offset + length)
+ *                (else GNMR_ERR_LAYOUT).
+ *   stream       cudaStream_t as void*; NULL = legacy default stream.
+ *   d_mask       device uint8 [num_units], written (1 = recovery path).
+ *   stats        optional statistics outputs (see gnmr_stats), or NULL.
+ * The arena must not change until the stream has passed the step.  Errors:
+ * GNMR_ERR_INVALID_ARG, GNMR_ERR_LAYOUT, GNMR_ERR_STATE, GNMR_ERR_CUDA (the
+ * launch failed). */
+gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems,
+                      void *stream, uint8_t *d_mask, const gnmr_stats *stats);
+
+/* Overrides alpha_t and beta_t for the following steps ("scheduled
+ * relaxation", Sec. 3.4).  NaN for either value returns it to the two-stage
+ * schedule.  Other values must be finite and > 0 (else
+ * GNMR_ERR_INVALID_ARG). */
+gnmr_status gnmr_set_thresholds(gnmr_handle *h, double alpha, double beta);
+
+/* Reports the launch geometry and memory of the handle into *info. */
+gnmr_status gnmr_get_info(const gnmr_handle *h, gnmr_info *info);
+
+/* Waits for work in flight on the handle's device, frees everything the handle owns and the
+ * handle itself.  NULL is accepted (GNMR_OK). */
+gnmr_status gnmr_destroy(gnmr_handle *h);
+
+/* Static text for a status code. */
+const char *gnmr_status_string(gnmr_status s);
+
+/* Detail of the last failure on h; with h == NULL, of the last failed
+ * gnmr_create on the calling thread.  Valid until the next call on h (or
+ * create on this thread); never NULL. */
+const char *gnmr_last_error(const gnmr_handle *h);
+
+/* Host-only query of the work partition that gnmr_create would plan: the
+ * concatenation of all units (an empty unit counts as one element of work)
+ * is cut into at most max_warps contiguous runs of about equal cost
+ * (element bytes plus a fixed per-unit cost), one run per warp.  Outputs,
+ * caller-allocated: run_unit / run_pos [max_warps + 1] (run w covers
+ * (run_unit[w], run_pos[w]) up to, not including, (run_unit[w+1],
+ * run_pos[w+1])), first_warp / num_parts [num_units] (the warps touching
+ * unit b are first_warp[b] .. first_warp[b] + num_parts[b] - 1).  *num_warps
+ * receives the number of runs.  No CUDA call is made.  Errors:
+ * GNMR_ERR_INVALID_ARG. */
+gnmr_status gnmr_plan_partition(int32_t num_units, const int64_t *lengths, int32_t dtype,
+                                int32_t max_warps, int32_t *num_warps, int32_t *run_unit,
+                                int64_t *run_pos, int32_t *first_warp, int32_t *num_parts);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GNMR_H */

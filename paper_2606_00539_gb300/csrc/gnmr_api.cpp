@@ -1,0 +1,407 @@
+// Host side of the libgnmr C ABI (include/gnmr.h): argument and layout
+// validation, the work plan, the single device allocation that holds all
+// library-owned state, and the per-step launch.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <limits>
+#include <new>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime_api.h>
+
+#include "gnmr.h"
+#include "gnmr_internal.h"
+
+struct gnmr_handle {
+    gnmr_config cfg{};            // layout pointers cleared after create
+    int32_t num_units = 0;
+    int elem_bytes = 0;
+    int32_t num_ctas = 0;
+    int32_t num_warps = 0;
+    int64_t num_partials = 0;
+    int64_t device_bytes = 0;
+    int64_t max_end = 0;
+    int64_t steps = 0;
+    double alpha_override = std::numeric_limits<double>::quiet_NaN();
+    double beta_override = std::numeric_limits<double>::quiet_NaN();
+    bool broken = false;
+    std::string err;
+    void *dmem = nullptr;
+    gnmr::StepParams params{};    // device pointers filled at create
+};
+
+namespace {
+
+thread_local std::string g_create_error;
+
+std::string format(const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    std::vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    return buf;
+}
+
+gnmr_status fail_create(gnmr_status s, const std::string &why)
+{
+    g_create_error = why;
+    return s;
+}
+
+gnmr_status fail(gnmr_handle *h, gnmr_status s, const std::string &why)
+{
+    h->err = why;
+    return s;
+}
+
+// Makes `dev` current for the scope of a call and restores the caller's.
+class DeviceScope {
+public:
+    explicit DeviceScope(int dev)
+    {
+        if (cudaGetDevice(&prev_) != cudaSuccess) {
+            prev_ = -1;
+            status_ = cudaErrorNoDevice;
+            return;
+        }
+        status_ = prev_ == dev ? cudaSuccess : cudaSetDevice(dev);
+    }
+    ~DeviceScope()
+    {
+        if (prev_ >= 0)
+            cudaSetDevice(prev_);
+    }
+    cudaError_t status() const { return status_; }
+
+private:
+    int prev_ = -1;
+    cudaError_t status_ = cudaSuccess;
+};
+
+bool positive_finite(double x) { return std::isfinite(x) && x > 0.0; }
+
+// Carves sub-buffers out of one allocation, each 256-byte aligned.
+struct Carver {
+    size_t size = 0;
+    size_t take(size_t bytes)
+    {
+        size_t at = size;
+        size += (bytes + 255) / 256 * 256;
+        return at;
+    }
+};
+
+}  // namespace
+
+extern "C" {
+
+void gnmr_config_defaults(gnmr_config *cfg)
+{
+    if (!cfg)
+        return;
+    std::memset(cfg, 0, sizeof *cfg);
+    cfg->dtype = GNMR_DTYPE_BF16;
+    cfg->window = 8;
+    cfg->max_o = 4;
+    cfg->lock_len = 1;
+    cfg->alpha_init = 1.5;
+    cfg->alpha_main = 1.1;
+    cfg->beta_init = 1.5;
+    cfg->beta_main = 1.5;
+    cfg->warmup_steps = 0;
+    cfg->eps = 1e-8;
+    cfg->device = 0;
+}
+
+const char *gnmr_status_string(gnmr_status s)
+{
+    switch (s) {
+    case GNMR_OK: return "GNMR_OK";
+    case GNMR_ERR_INVALID_ARG: return "GNMR_ERR_INVALID_ARG: invalid argument";
+    case GNMR_ERR_LAYOUT: return "GNMR_ERR_LAYOUT: unit layout does not fit the arena";
+    case GNMR_ERR_CUDA: return "GNMR_ERR_CUDA: CUDA call failed";
+    case GNMR_ERR_OOM: return "GNMR_ERR_OOM: out of memory";
+    case GNMR_ERR_STATE: return "GNMR_ERR_STATE: handle unusable after an earlier CUDA error";
+    }
+    return "unknown gnmr_status";
+}
+
+const char *gnmr_last_error(const gnmr_handle *h)
+{
+    return h ? h->err.c_str() : g_create_error.c_str();
+}
+
+gnmr_status gnmr_plan_partition(int32_t num_units, const int64_t *lengths, int32_t dtype,
+                                int32_t max_warps, int32_t *num_warps, int32_t *run_unit,
+                                int64_t *run_pos, int32_t *first_warp, int32_t *num_parts)
+{
+    if (num_units < 1 || !lengths || (dtype != GNMR_DTYPE_F32 && dtype != GNMR_DTYPE_BF16) ||
+        max_warps < 1 || !num_warps || !run_unit || !run_pos || !first_warp || !num_parts)
+        return GNMR_ERR_INVALID_ARG;
+    gnmr::Plan plan;
+    try {
+        if (!gnmr::plan_partition(num_units, lengths, dtype == GNMR_DTYPE_BF16 ? 2 : 4, max_warps, plan))
+            return GNMR_ERR_INVALID_ARG;
+    } catch (const std::bad_alloc &) {
+        return GNMR_ERR_OOM;
+    }
+    *num_warps = plan.num_warps;
+    std::memcpy(run_unit, plan.run_unit.data(), sizeof(int32_t) * (plan.num_warps + 1));
+    std::memcpy(run_pos, plan.run_pos.data(), sizeof(int64_t) * (plan.num_warps + 1));
+    std::memcpy(first_warp, plan.first_warp.data(), sizeof(int32_t) * num_units);
+    std::memcpy(num_parts, plan.num_parts.data(), sizeof(int32_t) * num_units);
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
+{
+    if (out)
+        *out = nullptr;
+    if (!cfg || !out)
+        return fail_create(GNMR_ERR_INVALID_ARG, "cfg and out must not be NULL");
+    const gnmr_config &c = *cfg;
+    if (c.num_units < 1)
+        return fail_create(GNMR_ERR_INVALID_ARG, format("num_units must be >= 1 (got %d)", c.num_units));
+    if (!c.offsets || !c.lengths)
+        return fail_create(GNMR_ERR_INVALID_ARG, "offsets and lengths must not be NULL");
+    if (c.dtype != GNMR_DTYPE_F32 && c.dtype != GNMR_DTYPE_BF16)
+        return fail_create(GNMR_ERR_INVALID_ARG, format("unknown dtype %d", c.dtype));
+    if (c.window < 1 || c.window > (1 << 16))
+        return fail_create(GNMR_ERR_INVALID_ARG, format("window must be in [1, 65536] (got %d)", c.window));
+    if (c.max_o < 0 || c.lock_len < 0 || c.warmup_steps < 0)
+        return fail_create(GNMR_ERR_INVALID_ARG, "max_o, lock_len and warmup_steps must be >= 0");
+    if (!positive_finite(c.alpha_init) || !positive_finite(c.alpha_main) ||
+        !positive_finite(c.beta_init) || !positive_finite(c.beta_main))
+        return fail_create(GNMR_ERR_INVALID_ARG, "thresholds alpha/beta must be finite and > 0");
+    if (!std::isfinite(c.eps) || c.eps < 0.0)
+        return fail_create(GNMR_ERR_INVALID_ARG, "eps must be finite and >= 0");
+    const int eb = c.dtype == GNMR_DTYPE_BF16 ? 2 : 4;
+    const int64_t limit = std::numeric_limits<int64_t>::max() / 8;
+    int64_t max_end = 0;
+    for (int32_t b = 0; b < c.num_units; ++b) {
+        const int64_t o = c.offsets[b], l = c.lengths[b];
+        if (o < 0 || l < 0 || o > limit - l)
+            return fail_create(GNMR_ERR_INVALID_ARG,
+                               format("unit %d: offset %lld / length %lld out of range", b,
+                                      (long long)o, (long long)l));
+        if (l > 0 && o + l > max_end)
+            max_end = o + l;
+    }
+
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev < 1)
+        return fail_create(GNMR_ERR_CUDA, "no CUDA device available");
+    if (c.device < 0 || c.device >= ndev)
+        return fail_create(GNMR_ERR_INVALID_ARG, format("device %d out of range (%d devices)", c.device, ndev));
+    DeviceScope scope(c.device);
+    if (scope.status() != cudaSuccess)
+        return fail_create(GNMR_ERR_CUDA, format("cudaSetDevice(%d): %s", c.device,
+                                                 cudaGetErrorString(scope.status())));
+    int sms = 0, per_sm = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
+    if (e == cudaSuccess)
+        e = gnmr::step_occupancy(c.dtype, &per_sm);
+    if (e != cudaSuccess || sms < 1 || per_sm < 1)
+        return fail_create(GNMR_ERR_CUDA, format("device query failed: %s", cudaGetErrorString(e)));
+
+    gnmr_handle *h = new (std::nothrow) gnmr_handle;
+    if (!h)
+        return fail_create(GNMR_ERR_OOM, "host allocation failed");
+    const int64_t U = c.num_units;
+    try {
+        gnmr::Plan plan;
+        if (!gnmr::plan_partition(c.num_units, c.lengths, eb, sms * per_sm * gnmr::kWarpsPerCta, plan)) {
+            delete h;
+            return fail_create(GNMR_ERR_INVALID_ARG, "work partition failed (sizes out of range)");
+        }
+        const int64_t W = plan.num_warps;
+        Carver cv;
+        const size_t o_off = cv.take(sizeof(int64_t) * U);
+        const size_t o_len = cv.take(sizeof(int64_t) * U);
+        const size_t o_rec = cv.take(U);
+        const size_t o_run_unit = cv.take(sizeof(int32_t) * (W + 1));
+        const size_t o_run_pos = cv.take(sizeof(int64_t) * (W + 1));
+        const size_t o_first = cv.take(sizeof(int32_t) * U);
+        const size_t o_parts = cv.take(sizeof(int32_t) * U);
+        const size_t o_pbase = cv.take(sizeof(int64_t) * U);
+        const size_t o_partial = cv.take(sizeof(double) * plan.num_partials);
+        const size_t o_ticket = cv.take(sizeof(uint32_t) * U);
+        const size_t o_state = cv.take(sizeof(gnmr::UnitState) * U);
+        const size_t o_queue = cv.take(sizeof(double) * U * c.window);
+        const size_t o_cand = cv.take(sizeof(gnmr::Candidate) * U);
+        const size_t o_ctl = cv.take(sizeof(gnmr::Control));
+
+        // Host image of the whole block: static tables plus zeroed state.
+        std::vector<unsigned char> img(cv.size, 0);
+        std::memcpy(&img[o_off], c.offsets, sizeof(int64_t) * U);
+        std::memcpy(&img[o_len], c.lengths, sizeof(int64_t) * U);
+        for (int64_t b = 0; b < U; ++b)
+            img[o_rec + b] = c.recoverable ? (c.recoverable[b] != 0) : 1;
+        std::memcpy(&img[o_run_unit], plan.run_unit.data(), sizeof(int32_t) * (W + 1));
+        std::memcpy(&img[o_run_pos], plan.run_pos.data(), sizeof(int64_t) * (W + 1));
+        std::memcpy(&img[o_first], plan.first_warp.data(), sizeof(int32_t) * U);
+        std::memcpy(&img[o_parts], plan.num_parts.data(), sizeof(int32_t) * U);
+        std::memcpy(&img[o_pbase], plan.part_base.data(), sizeof(int64_t) * U);
+
+        e = cudaMalloc(&h->dmem, cv.size);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            delete h;
+            return fail_create(e == cudaErrorMemoryAllocation ? GNMR_ERR_OOM : GNMR_ERR_CUDA,
+                               format("cudaMalloc(%zu): %s", cv.size, cudaGetErrorString(e)));
+        }
+        e = cudaMemcpy(h->dmem, img.data(), cv.size, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) {
+            cudaFree(h->dmem);
+            delete h;
+            return fail_create(GNMR_ERR_CUDA, format("cudaMemcpy: %s", cudaGetErrorString(e)));
+        }
+
+        char *base = static_cast<char *>(h->dmem);
+        gnmr::StepParams &p = h->params;
+        p.offset = reinterpret_cast<const int64_t *>(base + o_off);
+        p.length = reinterpret_cast<const int64_t *>(base + o_len);
+        p.recoverable = reinterpret_cast<const uint8_t *>(base + o_rec);
+        p.run_unit = reinterpret_cast<const int32_t *>(base + o_run_unit);
+        p.run_pos = reinterpret_cast<const int64_t *>(base + o_run_pos);
+        p.first_warp = reinterpret_cast<const int32_t *>(base + o_first);
+        p.num_parts = reinterpret_cast<const int32_t *>(base + o_parts);
+        p.part_base = reinterpret_cast<const int64_t *>(base + o_pbase);
+        p.partial = reinterpret_cast<double *>(base + o_partial);
+        p.unit_ticket = reinterpret_cast<uint32_t *>(base + o_ticket);
+        p.state = reinterpret_cast<gnmr::UnitState *>(base + o_state);
+        p.queue = reinterpret_cast<double *>(base + o_queue);
+        p.cand = reinterpret_cast<gnmr::Candidate *>(base + o_cand);
+        p.ctl = reinterpret_cast<gnmr::Control *>(base + o_ctl);
+        p.num_units = c.num_units;
+        p.num_warps = plan.num_warps;
+        p.window = c.window;
+        p.max_o = c.max_o;
+        p.lock_len = c.lock_len;
+        p.warmup_steps = c.warmup_steps;
+        p.alpha_init = c.alpha_init;
+        p.alpha_main = c.alpha_main;
+        p.beta_init = c.beta_init;
+        p.beta_main = c.beta_main;
+        p.eps = c.eps;
+
+        h->cfg = c;
+        h->cfg.offsets = nullptr;
+        h->cfg.lengths = nullptr;
+        h->cfg.recoverable = nullptr;
+        h->num_units = c.num_units;
+        h->elem_bytes = eb;
+        h->num_warps = plan.num_warps;
+        h->num_ctas = (plan.num_warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
+        h->num_partials = plan.num_partials;
+        h->device_bytes = static_cast<int64_t>(cv.size);
+        h->max_end = max_end;
+    } catch (const std::bad_alloc &) {
+        if (h->dmem)
+            cudaFree(h->dmem);
+        delete h;
+        return fail_create(GNMR_ERR_OOM, "host allocation failed while planning");
+    }
+    *out = h;
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems, void *stream,
+                      uint8_t *d_mask, const gnmr_stats *stats)
+{
+    if (!h)
+        return GNMR_ERR_INVALID_ARG;
+    if (h->broken)
+        return fail(h, GNMR_ERR_STATE, "an earlier step failed in CUDA; destroy the handle");
+    if (!d_mask)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_mask must not be NULL");
+    if (arena_elems < 0)
+        return fail(h, GNMR_ERR_INVALID_ARG, "arena_elems must be >= 0");
+    if (!d_arena && h->max_end > 0)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_arena is NULL but units are not empty");
+    if (reinterpret_cast<uintptr_t>(d_arena) % static_cast<uintptr_t>(h->elem_bytes) != 0)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_arena is not aligned to the element size");
+    if (arena_elems < h->max_end)
+        return fail(h, GNMR_ERR_LAYOUT,
+                    format("arena holds %lld elements but the layout needs %lld",
+                           (long long)arena_elems, (long long)h->max_end));
+    DeviceScope scope(h->cfg.device);
+    if (scope.status() != cudaSuccess)
+        return fail(h, GNMR_ERR_CUDA, format("cudaSetDevice: %s", cudaGetErrorString(scope.status())));
+
+    gnmr::StepParams p = h->params;
+    p.arena = d_arena;
+    p.mask = d_mask;
+    if (stats) {
+        p.out_norm = stats->norm;
+        p.out_gnmr = stats->gnmr;
+        p.out_dgnmr = stats->dgnmr;
+        p.out_risk = stats->risk;
+        p.out_lock = stats->lock;
+        p.out_counts = stats->counts;
+    }
+    p.alpha_override = h->alpha_override;
+    p.beta_override = h->beta_override;
+    const cudaError_t e = gnmr::launch_step(p, h->cfg.dtype, h->num_ctas,
+                                            static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        h->broken = true;
+        return fail(h, GNMR_ERR_CUDA, format("step launch: %s", cudaGetErrorString(e)));
+    }
+    h->steps += 1;
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_set_thresholds(gnmr_handle *h, double alpha, double beta)
+{
+    if (!h)
+        return GNMR_ERR_INVALID_ARG;
+    if ((!std::isnan(alpha) && !positive_finite(alpha)) || (!std::isnan(beta) && !positive_finite(beta)))
+        return fail(h, GNMR_ERR_INVALID_ARG, "thresholds must be finite and > 0, or NaN");
+    h->alpha_override = alpha;
+    h->beta_override = beta;
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_get_info(const gnmr_handle *h, gnmr_info *info)
+{
+    if (!h || !info)
+        return GNMR_ERR_INVALID_ARG;
+    info->num_units = h->num_units;
+    info->dtype = h->cfg.dtype;
+    info->device = h->cfg.device;
+    info->num_ctas = h->num_ctas;
+    info->threads_per_cta = gnmr::kThreads;
+    info->num_warps = h->num_warps;
+    info->num_partials = h->num_partials;
+    info->device_bytes = h->device_bytes;
+    info->arena_elems_min = h->max_end;
+    info->steps = h->steps;
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_destroy(gnmr_handle *h)
+{
+    if (!h)
+        return GNMR_OK;
+    gnmr_status st = GNMR_OK;
+    {
+        DeviceScope scope(h->cfg.device);
+        if (scope.status() == cudaSuccess) {
+            // cudaFree waits for work in flight on the device before freeing.
+            if (h->dmem && cudaFree(h->dmem) != cudaSuccess)
+                st = GNMR_ERR_CUDA;
+        } else {
+            st = GNMR_ERR_CUDA;
+        }
+    }
+    delete h;
+    return st;
+}
+
+}  // extern "C"

@@ -1,0 +1,101 @@
+// Internal declarations shared by the host API (gnmr_api.cpp, gnmr_plan.cpp)
+// and the device code (gnmr_kernels.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+#include <vector>
+
+#include <cuda_runtime_api.h>
+
+namespace gnmr {
+
+// Launch shape of the step kernel.  512 threads = 16 warps per CTA; the
+// kernel is compiled for two resident CTAs per SM (<= 64 registers/thread).
+constexpr int kThreads = 512;
+constexpr int kWarpsPerCta = kThreads / 32;
+constexpr int kMinCtasPerSm = 2;
+
+// Work partition: a unit costs its element bytes plus this many bytes of
+// equivalent fixed work (reduction, Algorithm 1 update, bookkeeping); runs
+// are cut at multiples of kSplitBytes inside a unit, and no run is planned
+// smaller than kMinRunBytes unless the whole problem is.
+constexpr int64_t kUnitCostBytes = 4096;
+constexpr int64_t kSplitBytes = 512;
+constexpr int64_t kMinRunBytes = 16384;
+
+// Persistent per-unit controller state (Algorithm 1 and 2), 32 bytes.
+struct UnitState {
+    double mean;      // A_b, historical mean of n_b
+    int64_t count;    // k_b, steps at which b was observed
+    int32_t fill;     // |Q_b|, valid entries of the GNMR queue (<= window)
+    int32_t head;     // ring position of the oldest queue entry once full
+    int32_t lock;     // Lock_b
+    int32_t pad;
+};
+
+// Candidate-pool entry written by the unit epilogue, read by the selection.
+struct Candidate {
+    double risk;      // R_{b,t}
+    int32_t unit;
+    int32_t pad;
+};
+
+// Device-resident step control block.
+struct Control {
+    uint32_t ctas_done;   // CTA completion ticket of the current launch
+    uint32_t n_cand;      // |C_t| appended so far
+    int64_t steps;        // completed steps (t of the last step)
+};
+
+struct StepParams {
+    const void *arena;
+    const int64_t *offset;       // [U]
+    const int64_t *length;       // [U]
+    const uint8_t *recoverable;  // [U]
+    const int32_t *run_unit;     // [W + 1]
+    const int64_t *run_pos;      // [W + 1]
+    const int32_t *first_warp;   // [U]
+    const int32_t *num_parts;    // [U]
+    const int64_t *part_base;    // [U] first partial slot of unit b
+    double *partial;             // [num_partials]
+    uint32_t *unit_ticket;       // [U]
+    UnitState *state;            // [U]
+    double *queue;               // [U * window] GNMR ring buffers
+    Candidate *cand;             // [U]
+    Control *ctl;
+    uint8_t *mask;               // [U], caller
+    double *out_norm, *out_gnmr, *out_dgnmr, *out_risk;  // caller, optional
+    int32_t *out_lock, *out_counts;                       // caller, optional
+    int32_t num_units;
+    int32_t num_warps;
+    int32_t window;
+    int32_t max_o;
+    int32_t lock_len;
+    int32_t pad;
+    int64_t warmup_steps;
+    double alpha_init, alpha_main, beta_init, beta_main, eps;
+    double alpha_override, beta_override;  // NaN = two-stage schedule
+};
+
+// Enqueues one step; returns the launch status.
+cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream);
+
+// Resident CTAs per SM of the step kernel for `dtype`.
+cudaError_t step_occupancy(int dtype, int *ctas_per_sm);
+
+// Host-side work partition (gnmr_plan.cpp).
+struct Plan {
+    int32_t num_warps = 0;
+    std::vector<int32_t> run_unit;    // [num_warps + 1]
+    std::vector<int64_t> run_pos;     // [num_warps + 1]
+    std::vector<int32_t> first_warp;  // [U]
+    std::vector<int32_t> num_parts;   // [U]
+    std::vector<int64_t> part_base;   // [U]
+    int64_t num_partials = 0;
+};
+
+// Returns false if the inputs are out of range.
+bool plan_partition(int32_t num_units, const int64_t *lengths, int elem_bytes,
+                    int32_t max_warps, Plan &out);
+
+}  // namespace gnmr

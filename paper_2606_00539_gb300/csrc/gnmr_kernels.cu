@@ -1,0 +1,483 @@
+// GNMR per-step monitor: one kernel launch per training step on sm_103a.
+//
+// Phase 1, every warp (the hot loop).  Each warp owns one contiguous run of
+// the unit stream planned by gnmr_plan.cpp.  For every unit segment in its
+// run it streams the gradient with 16-byte read-only loads (8 in flight per
+// lane, 4 KiB per warp per iteration), squares in fp32, sums blocks of 16
+// iterations in fp32 and the blocks in fp64, and all-reduces across the warp
+// with shuffles: n_b = ||g_b||_2 (Sec. 2, Eq. local_gradient).  No shared
+// memory, no block barrier on this path.
+//
+// Phase 2, the warp that completes unit b.  A unit split over several warps
+// collects their partial sums through fixed slots and a per-unit ticket; the
+// warp that takes the last ticket sums the slots in slot order (so the result
+// does not depend on timing) and runs the unit epilogue: Algorithm 1 (GNMR,
+// Delta-GNMR, incremental mean, window queue), the combined risk
+// R = max{GNMR/alpha_t, Delta-GNMR/beta_t} and the candidate test
+// R > 1 or Lock > 0 (Sec. 3.3), appending candidates to a compact list.
+//
+// Phase 3, the last CTA to finish (grid ticket).  Top_maxO over the
+// candidate list by an in-CTA radix select on the 96-bit key
+// (R descending, unit index ascending), then the lock bookkeeping of
+// Algorithm 2, the mask write, and the reset of the counters for the next
+// launch.  No CTA ever waits for another: the tickets decide who continues,
+// so the kernel cannot hang whatever the grid size or residency.
+#include <cstdint>
+
+#include <cuda_runtime.h>
+#include <math_constants.h>
+
+#include "gnmr_internal.h"
+
+namespace gnmr {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kUnroll = 8;   // 16-byte loads in flight per lane
+constexpr int kFlush = 16;   // main-loop iterations summed in fp32 before the fp64 add
+
+template <int DT> struct Elem;
+template <> struct Elem<0> {             // fp32
+    static constexpr int kBytes = 4;
+    static constexpr uint32_t kMagnitude = 0x7fffffffu;
+};
+template <> struct Elem<1> {             // bf16, two per 32-bit word
+    static constexpr int kBytes = 2;
+    static constexpr uint32_t kMagnitude = 0x7fff7fffu;
+};
+
+// 16-byte streaming load: non-coherent read-only path, no L1 allocation,
+// 256-byte L2 prefetch granularity.
+__device__ __forceinline__ uint4 ld_stream16(const uint4 *p)
+{
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+
+// One element as an fp32 bit pattern (bf16 is the upper half of an fp32).
+template <int DT> __device__ __forceinline__ uint32_t ld_elem_bits(const char *p);
+template <> __device__ __forceinline__ uint32_t ld_elem_bits<0>(const char *p)
+{
+    return __ldg(reinterpret_cast<const unsigned int *>(p));
+}
+template <> __device__ __forceinline__ uint32_t ld_elem_bits<1>(const char *p)
+{
+    return static_cast<uint32_t>(__ldg(reinterpret_cast<const unsigned short *>(p))) << 16;
+}
+
+// Sum of squares of the elements packed in one 16-byte vector, in fp32.
+template <int DT> __device__ __forceinline__ float vec_sumsq(const uint4 v);
+template <> __device__ __forceinline__ float vec_sumsq<0>(const uint4 v)
+{
+    const float a = __uint_as_float(v.x), b = __uint_as_float(v.y);
+    const float c = __uint_as_float(v.z), d = __uint_as_float(v.w);
+    return fmaf(d, d, fmaf(c, c, fmaf(b, b, a * a)));
+}
+template <> __device__ __forceinline__ float vec_sumsq<1>(const uint4 v)
+{
+    float s0 = 0.f, s1 = 0.f;
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float lo = __uint_as_float(w[i] << 16);
+        const float hi = __uint_as_float(w[i] & 0xffff0000u);
+        s0 = fmaf(lo, lo, s0);
+        s1 = fmaf(hi, hi, s1);
+    }
+    return s0 + s1;
+}
+
+__device__ __forceinline__ double warp_allreduce_sum(double v)
+{
+    // xor butterfly: both partners add the same two operands, so every lane
+    // ends with the same bits.
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+// Sum of squares of n elements at seg, by the whole warp.  Returns the sum
+// in every lane and sets `suspect` when fp32 squaring may have lost accuracy:
+// a nonzero segment whose sum is below 2^-100 (denormal squares) or above
+// 2^100 (possible fp32 overflow), or a NaN/Inf sum.
+template <int DT>
+__device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n, int lane,
+                                                     bool &suspect)
+{
+    constexpr int kEB = Elem<DT>::kBytes;
+    constexpr int kVE = 16 / kEB;
+    const uint32_t mis = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(seg) & 15u);
+    int64_t head = static_cast<int64_t>(((16u - mis) & 15u) / kEB);
+    head = head < n ? head : n;
+    const int64_t nvec = (n - head) / kVE;
+    const int64_t tail = n - head - nvec * kVE;
+
+    uint32_t bits = 0;
+    float blk = 0.f;
+    if (lane < head) {
+        const uint32_t w = ld_elem_bits<DT>(seg + lane * kEB);
+        const float x = __uint_as_float(w);
+        bits |= w;
+        blk = fmaf(x, x, blk);
+    }
+    if (lane < tail) {
+        const uint32_t w = ld_elem_bits<DT>(seg + (head + nvec * kVE + lane) * kEB);
+        const float x = __uint_as_float(w);
+        bits |= w;
+        blk = fmaf(x, x, blk);
+    }
+
+    const uint4 *v = reinterpret_cast<const uint4 *>(seg + head * kEB);
+    double acc = 0.0;
+    int64_t i = lane;
+    int cnt = 0;
+    for (; i + (kUnroll - 1) * 32 < nvec; i += kUnroll * 32) {
+        uint4 r[kUnroll];
+#pragma unroll
+        for (int j = 0; j < kUnroll; ++j)
+            r[j] = ld_stream16(v + i + j * 32);
+        float a[kUnroll];
+#pragma unroll
+        for (int j = 0; j < kUnroll; ++j) {
+            a[j] = vec_sumsq<DT>(r[j]);
+            bits |= (r[j].x | r[j].y) | (r[j].z | r[j].w);
+        }
+        blk += ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
+        if (++cnt == kFlush) {
+            acc += static_cast<double>(blk);
+            blk = 0.f;
+            cnt = 0;
+        }
+    }
+    // Fewer than kUnroll vectors left for this lane: one predicated batch.
+    {
+        uint4 r[kUnroll - 1];
+#pragma unroll
+        for (int j = 0; j < kUnroll - 1; ++j)
+            r[j] = (i + j * 32 < nvec) ? ld_stream16(v + i + j * 32) : make_uint4(0u, 0u, 0u, 0u);
+        float a = 0.f;
+#pragma unroll
+        for (int j = 0; j < kUnroll - 1; ++j) {
+            a += vec_sumsq<DT>(r[j]);
+            bits |= (r[j].x | r[j].y) | (r[j].z | r[j].w);
+        }
+        blk += a;
+    }
+    acc += static_cast<double>(blk);
+    acc = warp_allreduce_sum(acc);
+    bits = __reduce_or_sync(kFull, bits);
+    suspect = (bits & Elem<DT>::kMagnitude) != 0u && !(acc >= 0x1p-100 && acc <= 0x1p+100);
+    return acc;
+}
+
+// Exact-product fallback: each element squared in fp64 (exact for fp32 and
+// bf16 inputs) and summed in fp64.  Taken only for segments flagged suspect.
+template <int DT>
+__device__ __noinline__ double warp_segment_sumsq_f64(const char *seg, int64_t n, int lane)
+{
+    constexpr int kEB = Elem<DT>::kBytes;
+    double acc = 0.0;
+    for (int64_t i = lane; i < n; i += 32) {
+        const double x = static_cast<double>(__uint_as_float(ld_elem_bits<DT>(seg + i * kEB)));
+        acc = fma(x, x, acc);
+    }
+    return warp_allreduce_sum(acc);
+}
+
+__device__ __forceinline__ double pick_threshold(double override_value, int64_t t, int64_t warmup,
+                                                 double init_value, double main_value)
+{
+    if (!isnan(override_value))
+        return override_value;
+    return t <= warmup ? init_value : main_value;
+}
+
+// Unit epilogue, one lane: Algorithm 1, the combined risk of Sec. 3.3, the
+// statistics outputs and the candidate test of Algorithm 2.
+__device__ void unit_epilogue(const StepParams &p, int32_t b, double sumsq)
+{
+    const double n = sqrt(sumsq);
+    const int64_t t = __ldcg(&p.ctl->steps) + 1;
+    UnitState s = p.state[b];
+    double g, d;
+    if (!isfinite(n)) {
+        // Non-finite gradient: maximal risk, no change to A_b, Q_b, k_b.
+        g = CUDART_INF;
+        d = CUDART_INF;
+    } else {
+        double *Q = p.queue + static_cast<int64_t>(b) * p.window;
+        g = (s.count == 0 || s.mean == 0.0) ? 1.0 : n / (s.mean + p.eps);
+        if (s.fill == p.window) {
+            double q = 0.0;
+            int idx = s.head;                        // oldest entry first
+            for (int k = 0; k < p.window; ++k) {
+                q += Q[idx];
+                idx = (idx + 1 == p.window) ? 0 : idx + 1;
+            }
+            const double den = q / static_cast<double>(p.window) + p.eps;
+            d = (den == 0.0) ? (g > 0.0 ? CUDART_INF : 1.0) : g / den;
+        } else {
+            d = 1.0;
+        }
+        s.count += 1;
+        s.mean = s.mean + (n - s.mean) / static_cast<double>(s.count);
+        if (s.fill < p.window) {                     // still filling: head stays 0
+            Q[s.fill] = g;
+            s.fill += 1;
+        } else {                                     // overwrite the oldest
+            Q[s.head] = g;
+            s.head = (s.head + 1 == p.window) ? 0 : s.head + 1;
+        }
+        p.state[b].mean = s.mean;
+        p.state[b].count = s.count;
+        p.state[b].fill = s.fill;
+        p.state[b].head = s.head;
+    }
+    const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
+    const double beta = pick_threshold(p.beta_override, t, p.warmup_steps, p.beta_init, p.beta_main);
+    const double x = g / alpha, y = d / beta;
+    const double r = x > y ? x : y;
+
+    if (p.out_norm) p.out_norm[b] = n;
+    if (p.out_gnmr) p.out_gnmr[b] = g;
+    if (p.out_dgnmr) p.out_dgnmr[b] = d;
+    if (p.out_risk) p.out_risk[b] = r;
+
+    if (p.recoverable[b] && (r > 1.0 || s.lock > 0)) {
+        const uint32_t slot = atomicAdd(&p.ctl->n_cand, 1u);
+        if (slot < static_cast<uint32_t>(p.num_units)) {   // at most one entry per unit
+            p.cand[slot].risk = r;
+            p.cand[slot].unit = b;
+        }
+    } else {
+        // Not a candidate: Lock_b is already 0 and b stays on the low-cost path.
+        p.mask[b] = 0;
+        if (p.out_lock) p.out_lock[b] = 0;
+    }
+}
+
+// Called by the whole warp after it reduced its part of unit b.
+__device__ __forceinline__ void finish_part(const StepParams &p, int32_t b, int warp, double s,
+                                            int lane)
+{
+    const int32_t parts = p.num_parts[b];
+    if (parts > 1) {
+        const int64_t base = p.part_base[b];
+        uint32_t last = 0;
+        if (lane == 0) {
+            __stcg(&p.partial[base + (warp - p.first_warp[b])], s);
+            __threadfence();
+            last = atomicAdd(&p.unit_ticket[b], 1u) == static_cast<uint32_t>(parts - 1);
+        }
+        last = __shfl_sync(kFull, last, 0);
+        if (!last)
+            return;
+        __threadfence();
+        double acc = 0.0;
+        for (int32_t j = lane; j < parts; j += 32)
+            acc += __ldcg(&p.partial[base + j]);
+        s = warp_allreduce_sum(acc);
+        if (lane == 0)
+            p.unit_ticket[b] = 0;                    // ready for the next step
+    }
+    if (lane == 0)
+        unit_epilogue(p, b, s);
+}
+
+// Order-preserving keys: R >= 0 (never NaN), so its IEEE bits order like its
+// value; the low word ranks lower unit indices higher.
+__device__ __forceinline__ uint64_t risk_key(double r)
+{
+    return r == 0.0 ? 0ull : static_cast<uint64_t>(__double_as_longlong(r));
+}
+__device__ __forceinline__ uint32_t index_key(int32_t b, int32_t num_units)
+{
+    return static_cast<uint32_t>(num_units - 1 - b);
+}
+
+// K-th largest 96-bit key (risk_key : index_key) among the m candidates,
+// 1 <= K < m, by most-significant-digit radix select with 8-bit digits.
+// Returns the threshold: exactly K keys compare >= it.  All threads of the
+// CTA call this.
+__device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, uint32_t *hist,
+                             uint32_t *misc, uint64_t &thr_hi, uint32_t &thr_lo)
+{
+    const int lo_bits = p.num_units > 1 ? 32 - __clz(static_cast<uint32_t>(p.num_units - 1)) : 0;
+    const int lo_digits = (lo_bits + 7) / 8;
+    uint64_t pre_hi = 0, msk_hi = 0;
+    uint32_t pre_lo = 0, msk_lo = 0;
+    uint32_t r = K;
+    for (int dgt = 0; dgt < 8 + lo_digits; ++dgt) {
+        const bool in_hi = dgt < 8;
+        const int shift = in_hi ? 56 - 8 * dgt : 8 * (lo_digits - 1 - (dgt - 8));
+        for (int i = threadIdx.x; i < 256; i += blockDim.x)
+            hist[i] = 0;
+        __syncthreads();
+        for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+            const uint64_t hi = risk_key(__ldcg(&p.cand[i].risk));
+            const uint32_t lo = index_key(__ldcg(&p.cand[i].unit), p.num_units);
+            if ((hi & msk_hi) == pre_hi && (lo & msk_lo) == pre_lo) {
+                const uint32_t dig = in_hi ? static_cast<uint32_t>(hi >> shift) & 0xffu
+                                           : (lo >> shift) & 0xffu;
+                atomicAdd(&hist[dig], 1u);
+            }
+        }
+        __syncthreads();
+        if (threadIdx.x < 32) {
+            const int l = threadIdx.x;               // lane l owns buckets 255-8l down to 248-8l
+            uint32_t c8[8], sum = 0;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                c8[j] = hist[255 - 8 * l - j];
+                sum += c8[j];
+            }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t v = __shfl_up_sync(kFull, incl, o);
+                if (l >= o)
+                    incl += v;
+            }
+            const uint32_t excl = incl - sum;
+            if (excl < r && r <= incl) {             // exactly one lane
+                uint32_t above = excl;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    if (above + c8[j] >= r) {
+                        misc[1] = static_cast<uint32_t>(255 - 8 * l - j);
+                        misc[2] = r - above;
+                        misc[3] = c8[j];
+                        break;
+                    }
+                    above += c8[j];
+                }
+            }
+        }
+        __syncthreads();
+        const uint32_t bucket = misc[1];
+        const uint32_t in_bucket = misc[3];
+        r = misc[2];
+        if (in_hi) {
+            pre_hi |= static_cast<uint64_t>(bucket) << shift;
+            msk_hi |= 0xffull << shift;
+        } else {
+            pre_lo |= bucket << shift;
+            msk_lo |= 0xffu << shift;
+        }
+        __syncthreads();
+        if (in_bucket == r)                          // every key with this prefix is in
+            break;
+    }
+    thr_hi = pre_hi;
+    thr_lo = pre_lo;
+}
+
+// Last CTA: Top_maxO, Algorithm 2's lock bookkeeping, mask, counts, reset.
+__device__ void select_and_commit(const StepParams &p, uint32_t *hist, uint32_t *misc)
+{
+    uint32_t m = __ldcg(&p.ctl->n_cand);
+    m = m < static_cast<uint32_t>(p.num_units) ? m : static_cast<uint32_t>(p.num_units);
+    const uint32_t cap = static_cast<uint32_t>(p.max_o);
+    const uint32_t K = m < cap ? m : cap;
+    const bool take_all = m <= cap;
+    uint64_t thr_hi = 0;
+    uint32_t thr_lo = 0;
+    if (!take_all && K > 0)
+        radix_select(p, m, K, hist, misc, thr_hi, thr_lo);
+    for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+        const double r = __ldcg(&p.cand[i].risk);
+        const int32_t b = __ldcg(&p.cand[i].unit);
+        bool sel;
+        if (take_all) {
+            sel = true;
+        } else if (K == 0) {
+            sel = false;
+        } else {
+            const uint64_t hi = risk_key(r);
+            sel = hi > thr_hi || (hi == thr_hi && index_key(b, p.num_units) >= thr_lo);
+        }
+        const int32_t prev = __ldcg(&p.state[b].lock);
+        const int32_t next = !sel ? 0 : (r > 1.0 ? p.lock_len : (prev - 1 > 0 ? prev - 1 : 0));
+        p.state[b].lock = next;
+        p.mask[b] = sel ? 1 : 0;
+        if (p.out_lock) p.out_lock[b] = next;
+    }
+    if (threadIdx.x == 0 && p.out_counts) {
+        p.out_counts[0] = static_cast<int32_t>(m);
+        p.out_counts[1] = static_cast<int32_t>(K);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        p.ctl->n_cand = 0;
+        p.ctl->ctas_done = 0;
+        p.ctl->steps += 1;
+    }
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads, kMinCtasPerSm)
+gnmr_step_kernel(const __grid_constant__ StepParams p)
+{
+    __shared__ uint32_t s_hist[256];
+    __shared__ uint32_t s_misc[4];
+    constexpr int kEB = Elem<DT>::kBytes;
+    const int lane = threadIdx.x & 31;
+    const int warp = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+
+    if (warp < p.num_warps) {
+        int32_t b = p.run_unit[warp];
+        int64_t pos = p.run_pos[warp];
+        const int32_t b_end = p.run_unit[warp + 1];
+        const int64_t pos_end = p.run_pos[warp + 1];
+        const char *arena = static_cast<const char *>(p.arena);
+        while (b < b_end || (b == b_end && pos < pos_end)) {
+            const int64_t len = p.length[b];
+            int64_t stop = (b == b_end) ? pos_end : len;
+            stop = stop < len ? stop : len;
+            const int64_t n = stop > pos ? stop - pos : 0;
+            const char *seg = arena + (p.offset[b] + pos) * kEB;
+            bool suspect;
+            double s = warp_segment_sumsq<DT>(seg, n, lane, suspect);
+            if (suspect)
+                s = warp_segment_sumsq_f64<DT>(seg, n, lane);
+            finish_part(p, b, warp, s, lane);
+            ++b;
+            pos = 0;
+        }
+    }
+
+    // Grid completion: the last CTA through runs the selection.
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0)
+        s_misc[0] = atomicAdd(&p.ctl->ctas_done, 1u) == gridDim.x - 1 ? 1u : 0u;
+    __syncthreads();
+    if (s_misc[0]) {
+        __threadfence();
+        select_and_commit(p, s_hist, s_misc);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream)
+{
+    if (dtype == 1)
+        gnmr_step_kernel<1><<<num_ctas, kThreads, 0, stream>>>(p);
+    else
+        gnmr_step_kernel<0><<<num_ctas, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t step_occupancy(int dtype, int *ctas_per_sm)
+{
+    if (dtype == 1)
+        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<1>, kThreads, 0);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<0>, kThreads, 0);
+}
+
+}  // namespace gnmr

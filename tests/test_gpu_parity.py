@@ -1,0 +1,412 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Masks, locks and counts must match exactly; norms, GNMR, Delta-GNMR and R to
+a relative 1e-5.  The workloads run in lockstep with the oracle (see
+trace_driver) so that every rounded decision has margin."""
+import math
+from types import SimpleNamespace
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from paper_2606_00539_gb300 import Monitor
+from paper_2606_00539_gb300 import _native as N
+from tests import trace_driver as TD
+from tests.golden import hand_traces
+
+pytestmark = pytest.mark.gpu
+
+RTOL = 1e-5
+
+
+def _monitor(w, **over):
+    kw = w.monitor_kwargs()
+    kw.update(over)
+    return Monitor(w.offsets, w.lengths, device=0, **kw)
+
+
+def _run_lockstep(w, steps=None, every=1):
+    tr = TD.LockstepTrace(w, "cuda:0", _monitor)
+    try:
+        for t in range(steps or w.steps):
+            norms, res, got = tr.step(t)
+            if t % every == 0 or t == (steps or w.steps) - 1:
+                TD.compare(norms, res, got, RTOL)
+    finally:
+        tr.close()
+    return tr
+
+
+# ---------------------------------------------------------------------------
+# The five workloads (small cases: several tiles per unit and ragged tails)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("config,shrink,steps", [
+    ("tiny", 1, None),           # 64 fp32 units, 200 steps
+    ("llama2-1.3b", 8, 60),      # 168 bf16 units, dims / 8
+    ("llama2-13b", 16, None),    # 280 bf16 units, dims / 16, 20 steps
+    ("moe", 16, 30),             # 5454 bf16 units with unrouted experts
+    ("aq-stress", 1, 20),        # 100K fp32 units, contended top-64
+])
+def test_workload_parity(config, shrink, steps, cuda_device):
+    w = workloads.make(config, shrink=shrink, steps=steps)
+    tr = _run_lockstep(w)
+    assert sum(r.attempts for r in tr.records) < 10 * w.steps
+
+
+@pytest.mark.parametrize("seed", [1, 2])
+def test_tiny_more_seeds(seed, cuda_device):
+    _run_lockstep(workloads.make("tiny", seed=seed, steps=120))
+
+
+# ---------------------------------------------------------------------------
+# Hand-derived traces replayed on the GPU (exact norms: one fp32 element each)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("trace", hand_traces.all_traces(), ids=lambda t: t.name)
+def test_hand_trace_on_gpu(trace, cuda_device):
+    import torch
+    cfg = trace.cfg
+    U = int(cfg["units"])
+    off = np.arange(U, dtype=np.int64) * 4            # one element per unit, 16 B apart
+    ln = np.ones(U, np.int64)
+    mon = Monitor(off, ln, dtype="f32", recoverable=[int(x) for x in cfg["recoverable"]],
+                  window=int(cfg["window"]), max_o=int(cfg["max_o"]),
+                  lock_len=int(cfg["lock_len"]),
+                  alpha=(float(cfg["alpha_init"]), float(cfg["alpha_main"])),
+                  beta=(float(cfg["beta_init"]), float(cfg["beta_main"])),
+                  warmup_steps=int(cfg["warmup"]), eps=float(cfg["eps"]), device=0)
+    stats = mon.new_stats()
+    arena = torch.zeros(4 * U, dtype=torch.float32, device=cuda_device)
+    try:
+        for st in trace.steps:
+            arena[off] = torch.tensor([float(x) for x in st.n], dtype=torch.float32,
+                                      device=cuda_device)
+            mask = mon.step(arena, stats=stats).cpu().numpy()
+            g = {k: v.cpu().numpy() for k, v in stats.items()}
+            for b in range(U):
+                for key, want in (("gnmr", st.gnmr[b]), ("dgnmr", st.dgnmr[b]),
+                                  ("risk", st.risk[b])):
+                    want = float(want)
+                    if math.isinf(want):
+                        assert g[key][b] == want, (st.t, b, key)
+                    else:
+                        assert g[key][b] == pytest.approx(want, rel=1e-6, abs=1e-12), (st.t, b, key)
+            assert list(np.nonzero(mask)[0]) == st.selected, st.t
+            assert list(g["lock"]) == st.lock_after, st.t
+            assert list(g["counts"]) == [len(st.candidates), len(st.selected)], st.t
+    finally:
+        mon.close()
+
+
+# ---------------------------------------------------------------------------
+# Edge cases
+# ---------------------------------------------------------------------------
+
+def _random_arena(rng, n, dtype, scale=1.0):
+    import torch
+    x = torch.from_numpy((rng.standard_normal(n) * scale).astype(np.float32))
+    return x.to(torch.bfloat16) if dtype == "bf16" else x
+
+
+def _host_view(t):
+    import torch
+    t = t.cpu()
+    return t.view(torch.int16).numpy().view(np.uint16) if t.dtype == torch.bfloat16 else t.numpy()
+
+
+def _parity_on_norms(off, ln, dev_arena, make_step, mon_kw, ctl_kw, steps, recoverable=None):
+    """Runs `steps` steps.  make_step(t, attempt, bad) writes step t's
+    gradients into dev_arena; when the oracle finds a decision without margin
+    it is called again with attempt + 1 and the units to redraw (the oracle
+    state is rolled back first).  Every output is compared with the oracle."""
+    U = len(off)
+    rec = np.ones(U, np.uint8) if recoverable is None else np.asarray(recoverable, np.uint8)
+    mon = Monitor(off, ln, device=0, recoverable=rec, **mon_kw)
+    ctl = oracle.Controller(U, recoverable=rec, **ctl_kw)
+    stats = mon.new_stats()
+    margin_cfg = SimpleNamespace(recoverable=rec, warmup_steps=0,
+                                 **{k: ctl_kw[k] for k in ("alpha", "beta", "window", "max_o")})
+    try:
+        for t in range(steps):
+            attempt, bad = 0, []
+            while True:
+                make_step(t, attempt, bad)
+                norms = oracle.unit_norms(_host_view(dev_arena), off, ln)
+                before = ctl.get_state()
+                res = ctl.step(norms)
+                bad = TD.margin_violations(before, res, margin_cfg, t + 1)
+                if not bad:
+                    break
+                ctl.set_state(before)
+                attempt += 1
+                assert attempt < 30, f"no decision margin at step {t + 1}: units {bad[:8]}"
+            mask = mon.step(dev_arena, stats=stats)
+            got = {k: v.cpu().numpy() for k, v in stats.items()}
+            got["mask"] = mask.cpu().numpy()
+            TD.compare(norms, res, got, RTOL)
+    finally:
+        mon.close()
+        ctl.close()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_unaligned_overlapping_and_empty_units(dtype, cuda_device):
+    """Units at odd element offsets, overlapping units, gaps, zero-length and
+    one-element units, and a unit spanning many warps."""
+    import torch
+    rng = np.random.default_rng(11)
+    n = 3_000_001
+    off = np.array([0, 1, 3, 7, 100, 101, 5, 2_000_000, 17, 999_999, 0, 2_999_990], np.int64)
+    ln = np.array([1, 2, 13, 0, 1, 777, 2_000_000, 1_000_001, 0, 3, 3_000_001, 11], np.int64)
+    base = _random_arena(rng, n, "f32").to(cuda_device)
+    dev = torch.empty(n, dtype=torch.bfloat16 if dtype == "bf16" else torch.float32,
+                      device=cuda_device)
+    gen = torch.Generator(device=cuda_device)
+
+    def make_step(t, attempt, bad):
+        # fresh elementwise noise per step (and per attempt): every unit's
+        # norm moves on its own
+        gen.manual_seed(1000 * t + attempt)
+        noise = torch.randn(n, generator=gen, device=cuda_device)
+        x = base * (1.0 + 0.3 * noise)
+        if t == 3:
+            x[2_000_000:2_000_500] *= 40.0
+        dev.copy_(x.to(dev.dtype))
+
+    _parity_on_norms(off, ln, dev, make_step,
+                     dict(dtype=dtype, window=2, max_o=3, lock_len=2, alpha=1.2, beta=1.2),
+                     dict(window=2, max_o=3, lock_len=2, alpha=(1.2, 1.2), beta=(1.2, 1.2)), 6)
+
+
+def _per_unit_levels_arena(rng, ln, steps, sigma, device, zero_units=()):
+    """Packed fp32 units; step t of unit u is base * level[t, u].  Returns
+    (offsets, arena, make_step) with per-unit margin repair."""
+    import torch
+    off = np.concatenate([[0], np.cumsum(ln)[:-1]]).astype(np.int64)
+    base = _random_arena(rng, int(ln.sum()), "f32").to(device)
+    unit_of = torch.from_numpy(np.repeat(np.arange(len(ln)), ln)).to(device)
+    levels = np.exp(sigma * rng.standard_normal((steps, len(ln))))
+    for u in zero_units:
+        levels[:, u] = 0.0
+    dev = base.clone()
+    cur = {}
+
+    def make_step(t, attempt, bad):
+        if attempt == 0:
+            cur["lv"] = levels[t].copy()
+        for u in bad:
+            cur["lv"][u] *= math.exp(rng.uniform(-0.01, 0.01))
+        lv = torch.from_numpy(cur["lv"].astype(np.float32)).to(device)
+        dev.copy_(base * lv[unit_of])
+
+    return off, dev, make_step
+
+
+def test_nonfinite_gradients(cuda_device):
+    """NaN/Inf in a unit: R = +inf (selected first, ties by index), and the
+    unit's A, Q, k stay as they were -- checked over the following steps."""
+    rng = np.random.default_rng(13)
+    U, L = 16, 4096
+    ln = np.full(U, L, np.int64)
+    off, dev, base_step = _per_unit_levels_arena(rng, ln, 9, 0.2, cuda_device)
+
+    def make_step(t, attempt, bad):
+        base_step(t, attempt, bad)
+        if t == 4:
+            dev[5 * L + 17] = float("nan")
+            dev[9 * L + 3] = float("inf")
+            dev[2 * L + 100] = float("-inf")
+
+    _parity_on_norms(off, ln, dev, make_step,
+                     dict(dtype="f32", window=3, max_o=2, lock_len=1, alpha=1.5, beta=1.5),
+                     dict(window=3, max_o=2, lock_len=1, alpha=(1.5, 1.5), beta=(1.5, 1.5)), 9)
+
+
+@pytest.mark.parametrize("max_o,lock_len,thr", [(0, 3, 1.05), (10_000, 0, 1.05), (7, 2, 0.9)])
+def test_budget_extremes_and_ties(max_o, lock_len, thr, cuda_device):
+    """maxO = 0 (never select), maxO >= U (plain threshold), and thresholds
+    below 1 so that every unit ties at t = 1 (index order decides); some units
+    are not recoverable and some are all zeros."""
+    rng = np.random.default_rng(14)
+    U = 5000
+    ln = rng.integers(1, 300, U).astype(np.int64)
+    rec = (rng.random(U) < 0.9).astype(np.uint8)
+    off, dev, make_step = _per_unit_levels_arena(rng, ln, 8, 0.5, cuda_device,
+                                                 zero_units=range(0, U, 97))
+    _parity_on_norms(off, ln, dev, make_step,
+                     dict(dtype="f32", window=2, max_o=max_o, lock_len=lock_len, alpha=thr, beta=thr),
+                     dict(window=2, max_o=max_o, lock_len=lock_len, alpha=(thr, thr), beta=(thr, thr)),
+                     8, recoverable=rec)
+
+
+def test_tiny_and_huge_fp32_values_take_the_exact_path(cuda_device):
+    """fp32 squares underflow below ~1e-19 and overflow above ~1.8e19; the
+    kernel's fp64 fallback keeps the norm within rounding of the oracle."""
+    import torch
+    rng = np.random.default_rng(12)
+    parts = [rng.standard_normal(5000) * 1e-30, rng.standard_normal(5000) * 1e25,
+             rng.standard_normal(5000), np.concatenate([np.full(10, 1e-44), np.zeros(90)]),
+             rng.standard_normal(70000) * 3e-21]
+    host = np.concatenate(parts).astype(np.float32)
+    off = np.cumsum([0] + [len(p) for p in parts[:-1]]).astype(np.int64)
+    ln = np.array([len(p) for p in parts], np.int64)
+    dev = torch.from_numpy(host).to(cuda_device)
+    mon = Monitor(off, ln, dtype="f32", device=0)
+    stats = mon.new_stats()
+    try:
+        mon.step(dev, stats=stats)
+        got = stats["norm"].cpu().numpy()
+    finally:
+        mon.close()
+    want = oracle.unit_norms(host, off, ln)
+    assert np.all(want > 0)
+    np.testing.assert_allclose(got, want, rtol=RTOL, atol=0)
+
+
+def test_all_units_tie_under_contention(cuda_device):
+    """100K units, thresholds 0.5: at t = 1 every unit has R = 2; the top-64
+    must be units 0..63."""
+    import torch
+    U = 100_000
+    off = np.arange(U, dtype=np.int64) * 4
+    ln = np.full(U, 4, np.int64)
+    dev = torch.ones(4 * U, dtype=torch.float32, device=cuda_device)
+    mon = Monitor(off, ln, dtype="f32", max_o=64, lock_len=3, alpha=0.5, beta=0.5, window=4, device=0)
+    stats = mon.new_stats()
+    try:
+        mask = mon.step(dev, stats=stats).cpu().numpy()
+        assert list(np.nonzero(mask)[0]) == list(range(64))
+        assert list(stats["counts"].cpu().numpy()) == [U, 64]
+        assert np.all(stats["risk"].cpu().numpy() == 2.0)
+    finally:
+        mon.close()
+
+
+def test_threshold_override_and_schedule(cuda_device):
+    """gnmr_set_thresholds overrides alpha_t/beta_t until reset with NaN."""
+    w = workloads.make("tiny", seed=5, steps=40, shrink=8)
+    tr = TD.LockstepTrace(w, "cuda:0", _monitor)
+    try:
+        for t in range(w.steps):
+            if t == 20:
+                tr.mon.set_thresholds(1.05, 1.2)
+            if t == 30:
+                tr.mon.set_thresholds(float("nan"), float("nan"))
+            a, b = (1.05, 1.2) if 20 <= t < 30 else (math.nan, math.nan)
+            norms, res, got = tr.step(t, a, b)
+            TD.compare(norms, res, got, RTOL)
+    finally:
+        tr.close()
+
+
+def test_deterministic_across_handles_and_runs(cuda_device):
+    import torch
+    w = workloads.make("llama2-13b", shrink=32, steps=4)
+    f = workloads.Filler(w, cuda_device)
+    arena = f.new_arena()
+    outs = []
+    for _ in range(2):
+        mon = _monitor(w)
+        stats = mon.new_stats()
+        vals = []
+        for t in range(w.steps):
+            f.fill(arena, t)
+            mon.step(arena, stats=stats)
+            vals.append(stats["norm"].cpu().numpy().copy())
+        mon.close()
+        outs.append(np.stack(vals))
+    assert np.array_equal(outs[0].view(np.uint64), outs[1].view(np.uint64))
+
+
+def test_errors_leave_state_unchanged(cuda_device):
+    import torch
+    rng = np.random.default_rng(15)
+    U, L = 8, 1000
+    off = np.arange(U, dtype=np.int64) * L
+    ln = np.full(U, L, np.int64)
+    dev = _random_arena(rng, U * L, "bf16").to(cuda_device)
+    mon = Monitor(off, ln, dtype="bf16", device=0)
+    ctl = oracle.Controller(U, window=8, max_o=4, lock_len=1, alpha=(1.5, 1.1), beta=(1.5, 1.5))
+    stats = mon.new_stats()
+    mask = torch.empty(U, dtype=torch.uint8, device=cuda_device)
+    try:
+        h = mon._h
+        # arena shorter than the layout
+        with pytest.raises(N.GnmrError) as ei:
+            N.gnmr_step(h, dev.data_ptr(), U * L - 1, 0, mask.data_ptr(), None)
+        assert ei.value.status == N.GNMR_ERR_LAYOUT
+        # misaligned arena pointer (odd byte address for bf16)
+        with pytest.raises(N.GnmrError) as ei:
+            N.gnmr_step(h, dev.data_ptr() + 1, U * L, 0, mask.data_ptr(), None)
+        assert ei.value.status == N.GNMR_ERR_INVALID_ARG
+        with pytest.raises(N.GnmrError) as ei:
+            N.gnmr_step(h, dev.data_ptr(), U * L, 0, None, None)
+        assert ei.value.status == N.GNMR_ERR_INVALID_ARG
+        with pytest.raises(N.GnmrError):
+            mon.set_thresholds(-1.0, 1.0)
+        assert mon.info()["steps"] == 0
+        for t in range(3):
+            dev.mul_(1.0 + t)
+            norms = oracle.unit_norms(_host_view(dev), off, ln)
+            res = ctl.step(norms)
+            m = mon.step(dev, stats=stats)
+            got = {k: v.cpu().numpy() for k, v in stats.items()}
+            got["mask"] = m.cpu().numpy()
+            TD.compare(norms, res, got, RTOL)
+        assert mon.info()["steps"] == 3
+    finally:
+        mon.close()
+        ctl.close()
+
+
+def test_mask_only_and_side_stream(cuda_device):
+    import torch
+    w = workloads.make("tiny", seed=7, steps=12, shrink=4)
+    f = workloads.Filler(w, cuda_device)
+    arena = f.new_arena()
+    a = _monitor(w)
+    b = _monitor(w)
+    stats = b.new_stats()
+    side = torch.cuda.Stream(cuda_device)
+    try:
+        for t in range(w.steps):
+            f.fill(arena, t)
+            torch.cuda.synchronize()
+            with torch.cuda.stream(side):
+                m1 = a.step(arena, stream=side)
+            m2 = b.step(arena, stats=stats)
+            side.synchronize()
+            torch.cuda.synchronize()
+            assert torch.equal(m1, m2)
+    finally:
+        a.close()
+        b.close()
+
+
+def test_cuda_graph_replay_advances_steps(cuda_device):
+    """The step is one launch with no host synchronisation: captured once in a
+    CUDA graph and replayed, it matches the oracle step by step (the step
+    counter and thresholds live on the device)."""
+    import torch
+    w = workloads.make("tiny", seed=9, steps=30, shrink=4)
+    tr = TD.LockstepTrace(w, "cuda:0", _monitor)
+    mask = torch.empty(w.num_units, dtype=torch.uint8, device=cuda_device)
+    s = torch.cuda.Stream(cuda_device)
+    g = torch.cuda.CUDAGraph()
+    try:
+        with torch.cuda.graph(g, stream=s):
+            tr.mon.step(tr.arena, mask=mask, stats=tr.stats, stream=s)
+        # capturing does not run the kernel: the device state is still at t = 0
+
+        def replay():
+            g.replay()
+            return mask
+
+        for t in range(w.steps):
+            norms, res, got = tr.step(t, gpu_step=replay)
+            TD.compare(norms, res, got, RTOL)
+    finally:
+        tr.close()
