@@ -145,6 +145,22 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None}
 
 
+def profiled_traffic(kernel_source: str):
+    """DRAM bytes per launch from the committed ncu summary, or None once the
+    kernel source has changed since the counters were taken."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "gnmr_step_kernel_traffic.json")) as f:
+            rec = json.load(f)
+        with open(kernel_source, "rb") as f:
+            h = hashlib.sha256(f.read()).hexdigest()[:16]
+    except (OSError, ValueError):
+        return None
+    if rec.get("kernel_source_sha256_16") != h:
+        return None
+    return int(rec["traffic_bytes_per_launch"])
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -314,6 +330,7 @@ def run_gnmr(args):
     kern_ms = statistics.mean(per_ms)
     peak, peak_kind = measured_peaks()
     achieved = gbytes / (kern_ms / 1e3)
+    traffic = profiled_traffic(os.path.join(ROOT, "paper_2606_00539_gb300", "csrc", "gnmr_kernels.cu"))
 
     # end to end through the public API: host arena (pinned) -> device, the
     # step, the mask back to the host, every step inside the timed region
@@ -381,7 +398,10 @@ def run_gnmr(args):
                        "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
                                f"{info['num_warps']} warp runs"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
-                         "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                         "unit": "GB/s", "frac": round(achieved / peak, 4),
+                         "traffic": traffic if w.name == "llama2-13b" and args.shrink == 1 else None,
+                         "traffic_unit": "bytes per launch (ncu dram__bytes_read+write)",
+                         "algorithmic_bytes": w.grad_bytes,
                          "peak_source": f"{peak_kind} hbm_gbs", "kernel": "gnmr_step_kernel<bf16>",
                          "kernel_ms_mean": round(kern_ms, 4),
                          "kernel_ms_min": round(min(per_ms), 4)},
