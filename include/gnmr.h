@@ -159,7 +159,7 @@ gnmr_status gnmr_destroy(gnmr_handle *h);
 const char *gnmr_status_string(gnmr_status s);
 
 /* Detail of the last failure on h; with h == NULL, of the last failed
- * gnmr_create on the calling thread.  Valid until the next call on h (or
+ * gnmr_create or gnmr_unit_norms_static on the calling thread.  Valid until the next call on h (or
  * create on this thread); never NULL. */
 const char *gnmr_last_error(const gnmr_handle *h);
 
@@ -176,6 +176,43 @@ const char *gnmr_last_error(const gnmr_handle *h);
 gnmr_status gnmr_plan_partition(int32_t num_units, const int64_t *lengths, int32_t dtype,
                                 int32_t max_warps, int32_t *num_warps, int32_t *run_unit,
                                 int64_t *run_pos, int32_t *first_warp, int32_t *num_parts);
+
+/* Allocation-free per-unit norms.  The paper has no counterpart: this is a
+ * deployment variant of the first stage of gnmr_step.
+ *
+ * For callers that cannot allocate device memory -- code running inside a
+ * framework whose caching allocator already owns the GPU's memory, hooks
+ * called in the middle of a training step (where cudaMalloc/cudaFree would
+ * synchronise the device), deployments with a footprint fixed at start-up --
+ * and therefore cannot hold a gnmr_handle.  Computes n_b = ||g_b||_2 for
+ * every unit (the values gnmr_step writes to stats->norm) into d_norms, using
+ * as scratch only a device array that lives in the library's static data:
+ * about 11.5 MiB, reserved on every GPU that loads the library until the
+ * process exits.  No cudaMalloc, cudaFree or other allocating call is made.
+ *
+ * Arguments: d_arena (device, dtype elements, aligned to the element size;
+ * NULL only if every unit is empty), arena_elems, dtype (gnmr_dtype),
+ * num_units, offsets / lengths (HOST arrays of num_units elements, copied on
+ * the stream before the call returns), d_norms (device fp64 [num_units],
+ * written), stream (cudaStream_t as void*, NULL = legacy default stream).
+ * Runs on the calling thread's current device.
+ *
+ * Limits: num_units <= 131072 and sum over units of max(1, ceil(length
+ * bytes / 64 KiB)) <= 1048576 (so up to 64 GiB of gradient in large units);
+ * beyond them GNMR_ERR_INVALID_ARG, with gnmr_last_error(NULL) reading
+ * "units > 131072" or "chunks>1048576".  A unit outside [0, arena_elems)
+ * gives GNMR_ERR_LAYOUT ("unit off arena"); other details: "dtype unknown",
+ * "NULL pointer", "arena misalign", "CUDA failed".  The call makes no host
+ * allocation either, on success or failure.
+ *
+ * The first call on a device looks up the array's device address for that
+ * device; make that first call before any stream capture.  Every call shares
+ * the one array and leaves its contents behind (each call clears what must
+ * start at zero); calls that overlap on the GPU race on it, so callers must
+ * serialise them (one stream, one thread at a time). */
+gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena_elems, int32_t dtype,
+                                   int32_t num_units, const int64_t *offsets,
+                                   const int64_t *lengths, double *d_norms, void *stream);
 
 #ifdef __cplusplus
 }

@@ -89,6 +89,8 @@ PROTOTYPES = {
     "gnmr_last_error": (ctypes.c_char_p, [_P]),
     "gnmr_plan_partition": (ctypes.c_int, [ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int32,
                                            _P, _P, _P, _P, _P]),
+    "gnmr_unit_norms_static": (ctypes.c_int, [_P, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                              _P, _P, _P, _P]),
 }
 
 _lib = None

@@ -405,3 +405,12 @@ gnmr_status gnmr_destroy(gnmr_handle *h)
 }
 
 }  // extern "C"
+
+namespace gnmr {
+
+void record_thread_error(const char *why)
+{
+    g_create_error = why ? why : "";
+}
+
+}  // namespace gnmr

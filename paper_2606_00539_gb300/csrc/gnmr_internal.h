@@ -83,6 +83,10 @@ cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream
 // Resident CTAs per SM of the step kernel for `dtype`.
 cudaError_t step_occupancy(int dtype, int *ctas_per_sm);
 
+// Records the failure detail that gnmr_last_error(NULL) reports on the
+// calling thread (used by calls that have no handle).
+void record_thread_error(const char *why);
+
 // Host-side work partition (gnmr_plan.cpp).
 struct Plan {
     int32_t num_warps = 0;
