@@ -46,6 +46,8 @@ def parse_args(argv=None):
                    help="divide matrix dims (small case for profiler captures)")
     p.add_argument("--arenas", type=int, default=2, help="distinct step arenas cycled")
     p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--flush-l2", action="store_true",
+                   help="write 512 MB before every timed step (outside its events)")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-units", type=int, default=0,
@@ -73,6 +75,11 @@ def max_over_ranks(value: float, world: int, device=None) -> float:
     t = torch.tensor([value], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def throughput_gbs(world: int, bytes_per_step: int, steps: int, max_ms: float) -> float:
+    """Whole-job GB/s: every rank's gradient bytes over the slowest rank's time."""
+    return world * bytes_per_step * steps / (max_ms / 1e3) / 1e9
 
 
 def barrier(world: int, device=None):
@@ -283,8 +290,9 @@ def run_gnmr(args):
     n_arenas = max(1, args.arenas)
     arenas = []
     for i in range(n_arenas):
+        # steps from the middle of the trace: spikes, ramps and locks are live
         a = filler.new_arena()
-        filler.fill(a, i % w.steps)
+        filler.fill(a, (w.steps // 2 + i) % w.steps)
         arenas.append(a)
     mon = Monitor(w.offsets, w.lengths, device=local_rank, **w.monitor_kwargs())
     info = mon.info()
@@ -306,8 +314,12 @@ def run_gnmr(args):
     barrier(world, dev)
     torch.cuda.synchronize(dev)
     wall0 = time.time()
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if args.flush_l2 else None
     t_start.record(stream)
     for i in range(args.steps):
+        if flush is not None:
+            with torch.cuda.stream(stream):
+                flush.zero_()
         ev[i][0].record(stream)
         mon.step(arenas[(args.warmup + i) % n_arenas], mask=mask, stats=stats, stream=stream)
         ev[i][1].record(stream)
@@ -319,13 +331,14 @@ def run_gnmr(args):
     sampler.stop()
     clocks = sampler.summary(wall0, wall1)
 
-    total_ms = t_start.elapsed_time(t_end)
     per_ms = [a.elapsed_time(b) for a, b in ev]
+    # with flushes in the region, the step time is the sum of the steps' own events
+    total_ms = sum(per_ms) if flush is not None else t_start.elapsed_time(t_end)
     max_ms = max_over_ranks(total_ms, world, dev)
     launches = args.steps                              # one kernel per gnmr_step
 
     gbytes = w.grad_bytes / 1e9
-    value = world * gbytes * args.steps / (max_ms / 1e3)
+    value = throughput_gbs(world, w.grad_bytes, args.steps, max_ms)
     step_ms = max_ms / args.steps
     kern_ms = statistics.mean(per_ms)
     peak, peak_kind = measured_peaks()
@@ -392,8 +405,9 @@ def run_gnmr(args):
             "config": {"workload": f"{w.name} ({w.num_units} units, {w.grad_elems} {w.dtype} "
                                    f"elements{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
                        "bytes_per_step": w.grad_bytes, "arenas_cycled": n_arenas,
-                       "l2": "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * 129e6
-                       else "inputs fit in L2 (hot)",
+                       "l2": ("L2 flushed before every step (512 MB write)" if args.flush_l2
+                              else "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * 129e6
+                              else "inputs fit in L2 (hot)"),
                        "parallelism": "replicas" if world > 1 else "single GPU",
                        "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
                                f"{info['num_warps']} warp runs"},
@@ -402,7 +416,7 @@ def run_gnmr(args):
                          "traffic": traffic if w.name == "llama2-13b" and args.shrink == 1 else None,
                          "traffic_unit": "bytes per launch (ncu dram__bytes_read+write)",
                          "algorithmic_bytes": w.grad_bytes,
-                         "peak_source": f"{peak_kind} hbm_gbs", "kernel": "gnmr_step_kernel<bf16>",
+                         "peak_source": f"{peak_kind} hbm_gbs", "kernel": f"gnmr_step_kernel<{w.dtype}>",
                          "kernel_ms_mean": round(kern_ms, 4),
                          "kernel_ms_min": round(min(per_ms), 4)},
             "cpu_baseline": cpu,

@@ -33,11 +33,12 @@ struct UnitState {
     int32_t pad;
 };
 
-// Candidate-pool entry written by the unit epilogue, read by the selection.
+// Candidate-pool entry written by the unit epilogue, read by the selection
+// (one 16-byte load).
 struct Candidate {
     double risk;      // R_{b,t}
     int32_t unit;
-    int32_t pad;
+    int32_t lock;     // Lock_b before this step
 };
 
 // Device-resident step control block.

@@ -11,8 +11,9 @@
 // Phase 2, the warp that completes unit b.  A unit split over several warps
 // collects their partial sums through fixed slots and a per-unit ticket; the
 // warp that takes the last ticket sums the slots in slot order (so the result
-// does not depend on timing) and runs the unit epilogue: Algorithm 1 (GNMR,
-// Delta-GNMR, incremental mean, window queue), the combined risk
+// does not depend on timing).  Completed units queue up in the warp's lanes
+// and run the unit epilogue 32 at a time, one unit per lane: Algorithm 1
+// (GNMR, Delta-GNMR, incremental mean, window queue), the combined risk
 // R = max{GNMR/alpha_t, Delta-GNMR/beta_t} and the candidate test
 // R > 1 or Lock > 0 (Sec. 3.3), appending candidates to a compact list.
 //
@@ -196,96 +197,128 @@ __device__ __forceinline__ double pick_threshold(double override_value, int64_t 
     return t <= warmup ? init_value : main_value;
 }
 
-// Unit epilogue, one lane: Algorithm 1, the combined risk of Sec. 3.3, the
-// statistics outputs and the candidate test of Algorithm 2.
-__device__ void unit_epilogue(const StepParams &p, int32_t b, double sumsq)
+// Unit epilogue for up to 32 units at once, one per lane (lanes with
+// `active` false only take part in the collective append): Algorithm 1, the
+// combined risk of Sec. 3.3, the statistics outputs and the candidate test of
+// Algorithm 2.  Every lane issues its unit's loads together, so a batch costs
+// about one memory round trip; candidates are appended with one atomic per
+// warp.  Called by all 32 lanes.
+__device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, double sumsq,
+                              double alpha, double beta)
 {
-    const double n = sqrt(sumsq);
-    const int64_t t = __ldcg(&p.ctl->steps) + 1;
-    UnitState s = p.state[b];
-    double g, d;
-    if (!isfinite(n)) {
-        // Non-finite gradient: maximal risk, no change to A_b, Q_b, k_b.
-        g = CUDART_INF;
-        d = CUDART_INF;
-    } else {
-        double *Q = p.queue + static_cast<int64_t>(b) * p.window;
-        g = (s.count == 0 || s.mean == 0.0) ? 1.0 : n / (s.mean + p.eps);
-        if (s.fill == p.window) {
-            double q = 0.0;
-            int idx = s.head;                        // oldest entry first
-            for (int k = 0; k < p.window; ++k) {
-                q += Q[idx];
-                idx = (idx + 1 == p.window) ? 0 : idx + 1;
-            }
-            const double den = q / static_cast<double>(p.window) + p.eps;
-            d = (den == 0.0) ? (g > 0.0 ? CUDART_INF : 1.0) : g / den;
+    bool cand = false;
+    double r = 0.0;
+    int32_t lock_prev = 0;
+    if (active) {
+        const double n = sqrt(sumsq);
+        UnitState s = p.state[b];
+        double g, d;
+        if (!isfinite(n)) {
+            // Non-finite gradient: maximal risk, no change to A_b, Q_b, k_b.
+            g = CUDART_INF;
+            d = CUDART_INF;
         } else {
-            d = 1.0;
+            const int w = p.window;
+            double *Q = p.queue + static_cast<int64_t>(b) * w;
+            g = (s.count == 0 || s.mean == 0.0) ? 1.0 : n / (s.mean + p.eps);
+            if (s.fill == w) {
+                // mean of the window, summed oldest to newest; loads issued 8 at a time
+                double q = 0.0;
+                int idx = s.head, k = 0;
+                for (; k + 8 <= w; k += 8) {
+                    double v[8];
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const int ix = idx + j < w ? idx + j : idx + j - w;
+                        v[j] = Q[ix];
+                    }
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        q += v[j];
+                    idx = idx + 8 < w ? idx + 8 : idx + 8 - w;
+                }
+                for (; k < w; ++k) {
+                    q += Q[idx];
+                    idx = (idx + 1 == w) ? 0 : idx + 1;
+                }
+                const double den = q / static_cast<double>(w) + p.eps;
+                d = (den == 0.0) ? (g > 0.0 ? CUDART_INF : 1.0) : g / den;
+            } else {
+                d = 1.0;
+            }
+            s.count += 1;
+            s.mean = s.mean + (n - s.mean) / static_cast<double>(s.count);
+            if (s.fill < w) {                        // still filling: head stays 0
+                Q[s.fill] = g;
+                s.fill += 1;
+            } else {                                 // overwrite the oldest
+                Q[s.head] = g;
+                s.head = (s.head + 1 == w) ? 0 : s.head + 1;
+            }
+            p.state[b].mean = s.mean;
+            p.state[b].count = s.count;
+            p.state[b].fill = s.fill;
+            p.state[b].head = s.head;
         }
-        s.count += 1;
-        s.mean = s.mean + (n - s.mean) / static_cast<double>(s.count);
-        if (s.fill < p.window) {                     // still filling: head stays 0
-            Q[s.fill] = g;
-            s.fill += 1;
-        } else {                                     // overwrite the oldest
-            Q[s.head] = g;
-            s.head = (s.head + 1 == p.window) ? 0 : s.head + 1;
+        const double x = g / alpha, y = d / beta;
+        r = x > y ? x : y;
+
+        if (p.out_norm) p.out_norm[b] = n;
+        if (p.out_gnmr) p.out_gnmr[b] = g;
+        if (p.out_dgnmr) p.out_dgnmr[b] = d;
+        if (p.out_risk) p.out_risk[b] = r;
+
+        lock_prev = s.lock;
+        cand = p.recoverable[b] && (r > 1.0 || s.lock > 0);
+        if (!cand) {
+            // Not a candidate: Lock_b is already 0 and b stays on the low-cost path.
+            p.mask[b] = 0;
+            if (p.out_lock) p.out_lock[b] = 0;
         }
-        p.state[b].mean = s.mean;
-        p.state[b].count = s.count;
-        p.state[b].fill = s.fill;
-        p.state[b].head = s.head;
     }
-    const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
-    const double beta = pick_threshold(p.beta_override, t, p.warmup_steps, p.beta_init, p.beta_main);
-    const double x = g / alpha, y = d / beta;
-    const double r = x > y ? x : y;
-
-    if (p.out_norm) p.out_norm[b] = n;
-    if (p.out_gnmr) p.out_gnmr[b] = g;
-    if (p.out_dgnmr) p.out_dgnmr[b] = d;
-    if (p.out_risk) p.out_risk[b] = r;
-
-    if (p.recoverable[b] && (r > 1.0 || s.lock > 0)) {
-        const uint32_t slot = atomicAdd(&p.ctl->n_cand, 1u);
-        if (slot < static_cast<uint32_t>(p.num_units)) {   // at most one entry per unit
-            p.cand[slot].risk = r;
-            p.cand[slot].unit = b;
+    const unsigned want = __ballot_sync(kFull, cand);
+    if (want) {
+        const int lane = threadIdx.x & 31;
+        const int leader = __ffs(want) - 1;
+        uint32_t base = 0;
+        if (lane == leader)
+            base = atomicAdd(&p.ctl->n_cand, static_cast<uint32_t>(__popc(want)));
+        base = __shfl_sync(kFull, base, leader);
+        if (cand) {
+            const uint32_t slot = base + __popc(want & ((1u << lane) - 1u));
+            if (slot < static_cast<uint32_t>(p.num_units)) {   // at most one entry per unit
+                p.cand[slot].risk = r;
+                p.cand[slot].unit = b;
+                p.cand[slot].lock = lock_prev;
+            }
         }
-    } else {
-        // Not a candidate: Lock_b is already 0 and b stays on the low-cost path.
-        p.mask[b] = 0;
-        if (p.out_lock) p.out_lock[b] = 0;
     }
 }
 
-// Called by the whole warp after it reduced its part of unit b.
-__device__ __forceinline__ void finish_part(const StepParams &p, int32_t b, int warp, double s,
-                                            int lane)
+// A unit split over several warps: stores this warp's partial and takes a
+// ticket.  Returns true (with the unit's total in s) for the warp that takes
+// the last ticket; that warp sums the partials in slot order.
+__device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, int32_t parts, int warp,
+                                              double &s, int lane)
 {
-    const int32_t parts = p.num_parts[b];
-    if (parts > 1) {
-        const int64_t base = p.part_base[b];
-        uint32_t last = 0;
-        if (lane == 0) {
-            __stcg(&p.partial[base + (warp - p.first_warp[b])], s);
-            __threadfence();
-            last = atomicAdd(&p.unit_ticket[b], 1u) == static_cast<uint32_t>(parts - 1);
-        }
-        last = __shfl_sync(kFull, last, 0);
-        if (!last)
-            return;
+    const int64_t base = p.part_base[b];
+    uint32_t last = 0;
+    if (lane == 0) {
+        __stcg(&p.partial[base + (warp - p.first_warp[b])], s);
         __threadfence();
-        double acc = 0.0;
-        for (int32_t j = lane; j < parts; j += 32)
-            acc += __ldcg(&p.partial[base + j]);
-        s = warp_allreduce_sum(acc);
-        if (lane == 0)
-            p.unit_ticket[b] = 0;                    // ready for the next step
+        last = atomicAdd(&p.unit_ticket[b], 1u) == static_cast<uint32_t>(parts - 1);
     }
+    last = __shfl_sync(kFull, last, 0);
+    if (!last)
+        return false;
+    __threadfence();
+    double acc = 0.0;
+    for (int32_t j = lane; j < parts; j += 32)
+        acc += __ldcg(&p.partial[base + j]);
+    s = warp_allreduce_sum(acc);
     if (lane == 0)
-        unit_epilogue(p, b, s);
+        p.unit_ticket[b] = 0;                        // ready for the next step
+    return true;
 }
 
 // Order-preserving keys: R >= 0 (never NaN), so its IEEE bits order like its
@@ -297,6 +330,15 @@ __device__ __forceinline__ uint64_t risk_key(double r)
 __device__ __forceinline__ uint32_t index_key(int32_t b, int32_t num_units)
 {
     return static_cast<uint32_t>(num_units - 1 - b);
+}
+
+__device__ __forceinline__ void load_candidate(const Candidate *c, double &r, int32_t &b, int32_t &lock)
+{
+    const double2 v = __ldcg(reinterpret_cast<const double2 *>(c));
+    const uint64_t w = static_cast<uint64_t>(__double_as_longlong(v.y));
+    r = v.x;
+    b = static_cast<int32_t>(w & 0xffffffffu);
+    lock = static_cast<int32_t>(w >> 32);
 }
 
 // K-th largest 96-bit key (risk_key : index_key) among the m candidates,
@@ -317,13 +359,26 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, uint32
         for (int i = threadIdx.x; i < 256; i += blockDim.x)
             hist[i] = 0;
         __syncthreads();
-        for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
-            const uint64_t hi = risk_key(__ldcg(&p.cand[i].risk));
-            const uint32_t lo = index_key(__ldcg(&p.cand[i].unit), p.num_units);
-            if ((hi & msk_hi) == pre_hi && (lo & msk_lo) == pre_lo) {
-                const uint32_t dig = in_hi ? static_cast<uint32_t>(hi >> shift) & 0xffu
-                                           : (lo >> shift) & 0xffu;
-                atomicAdd(&hist[dig], 1u);
+        for (uint32_t i0 = threadIdx.x; i0 < m; i0 += 4 * blockDim.x) {
+            double rr[4];
+            int32_t bb[4], ll[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {           // four loads in flight per thread
+                const uint32_t i = i0 + j * blockDim.x;
+                if (i < m)
+                    load_candidate(p.cand + i, rr[j], bb[j], ll[j]);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if (i0 + j * blockDim.x >= m)
+                    break;
+                const uint64_t hi = risk_key(rr[j]);
+                const uint32_t lo = index_key(bb[j], p.num_units);
+                if ((hi & msk_hi) == pre_hi && (lo & msk_lo) == pre_lo) {
+                    const uint32_t dig = in_hi ? static_cast<uint32_t>(hi >> shift) & 0xffu
+                                               : (lo >> shift) & 0xffu;
+                    atomicAdd(&hist[dig], 1u);
+                }
             }
         }
         __syncthreads();
@@ -389,8 +444,9 @@ __device__ void select_and_commit(const StepParams &p, uint32_t *hist, uint32_t 
     if (!take_all && K > 0)
         radix_select(p, m, K, hist, misc, thr_hi, thr_lo);
     for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
-        const double r = __ldcg(&p.cand[i].risk);
-        const int32_t b = __ldcg(&p.cand[i].unit);
+        double r;
+        int32_t b, prev;
+        load_candidate(p.cand + i, r, b, prev);
         bool sel;
         if (take_all) {
             sel = true;
@@ -400,7 +456,6 @@ __device__ void select_and_commit(const StepParams &p, uint32_t *hist, uint32_t 
             const uint64_t hi = risk_key(r);
             sel = hi > thr_hi || (hi == thr_hi && index_key(b, p.num_units) >= thr_lo);
         }
-        const int32_t prev = __ldcg(&p.state[b].lock);
         const int32_t next = !sel ? 0 : (r > 1.0 ? p.lock_len : (prev - 1 > 0 ? prev - 1 : 0));
         p.state[b].lock = next;
         p.mask[b] = sel ? 1 : 0;
@@ -429,13 +484,23 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     const int warp = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
 
     if (warp < p.num_warps) {
+        // t, alpha_t and beta_t are fixed for the whole step.
+        const int64_t t = __ldcg(&p.ctl->steps) + 1;
+        const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
+        const double beta = pick_threshold(p.beta_override, t, p.warmup_steps, p.beta_init, p.beta_main);
         int32_t b = p.run_unit[warp];
         int64_t pos = p.run_pos[warp];
         const int32_t b_end = p.run_unit[warp + 1];
         const int64_t pos_end = p.run_pos[warp + 1];
         const char *arena = static_cast<const char *>(p.arena);
+        // Units this warp completes wait here, lane j holding the j-th, and run
+        // their epilogues 32 at a time.
+        int32_t pend_b = 0;
+        double pend_s = 0.0;
+        int npend = 0;
         while (b < b_end || (b == b_end && pos < pos_end)) {
             const int64_t len = p.length[b];
+            const int32_t parts = p.num_parts[b];
             int64_t stop = (b == b_end) ? pos_end : len;
             stop = stop < len ? stop : len;
             const int64_t n = stop > pos ? stop - pos : 0;
@@ -444,10 +509,21 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
             double s = warp_segment_sumsq<DT>(seg, n, lane, suspect);
             if (suspect)
                 s = warp_segment_sumsq_f64<DT>(seg, n, lane);
-            finish_part(p, b, warp, s, lane);
+            if (parts == 1 || combine_parts(p, b, parts, warp, s, lane)) {
+                if (lane == npend) {
+                    pend_b = b;
+                    pend_s = s;
+                }
+                if (++npend == 32) {
+                    unit_epilogue(p, true, pend_b, pend_s, alpha, beta);
+                    npend = 0;
+                }
+            }
             ++b;
             pos = 0;
         }
+        if (npend > 0)
+            unit_epilogue(p, lane < npend, pend_b, pend_s, alpha, beta);
     }
 
     // Grid completion: the last CTA through runs the selection.

@@ -82,6 +82,11 @@ class LockstepTrace:
         self.stats = self.mon.new_stats()
         self.threads = threads or min(16, os.cpu_count() or 1)
         self.records = []
+        self._pinned = None
+        if self.arena.numel() * self.arena.element_size() > (256 << 20):
+            # large arenas: one reusable pinned host copy instead of a fresh
+            # pageable allocation every step
+            self._pinned = torch.empty(self.arena.numel(), dtype=self.arena.dtype, pin_memory=True)
 
     def close(self):
         self.mon.close()
@@ -92,7 +97,11 @@ class LockstepTrace:
         w = self.w
         torch.cuda.synchronize(self.dev)
         if units is None:
-            host = self.arena.cpu()
+            if self._pinned is not None:
+                self._pinned.copy_(self.arena)
+                host = self._pinned
+            else:
+                host = self.arena.cpu()
             view = host.view(torch.int16).numpy().view(np.uint16) if w.dtype == "bf16" else host.numpy()
             return oracle.unit_norms_threaded(view, w.offsets, w.lengths, self.threads)
         out = {}
