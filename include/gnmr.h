@@ -142,6 +142,46 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out);
 gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems,
                       void *stream, uint8_t *d_mask, const gnmr_stats *stats);
 
+/* Sharded step, first half: this rank's per-unit sums of squares.
+ *
+ * With ZeRO-style sharded data parallelism each rank holds a slice of every
+ * unit's gradient, and n_b = ||g_b||_2 needs the sum of the slices' sums of
+ * squares (Eq. local_gradient).  The handle is created with the rank's local
+ * layout (a unit with no elements on this rank has length 0).  This call
+ * reads the local arena like gnmr_step but only writes
+ * d_sumsq[b] = sum of g_i^2 over unit b's local elements (device fp64
+ * [num_units]); it changes no controller state.  The caller then sums d_sumsq
+ * across ranks (e.g. an all-reduce) and calls gnmr_finish on every rank:
+ * identical sums give identical masks everywhere.  Arguments and errors as
+ * gnmr_step (d_sumsq replaces d_mask). */
+gnmr_status gnmr_step_partials(gnmr_handle *h, const void *d_arena, int64_t arena_elems,
+                               void *stream, double *d_sumsq);
+
+/* Sharded step, second half: one controller step (Algorithms 1 and 2, as in
+ * gnmr_step from step 2 on) on given per-unit sums of squares: n_b =
+ * sqrt(d_sumsq[b]).  d_sumsq: device fp64 [num_units], read only.  d_mask and
+ * stats as in gnmr_step.  Advances the step counter.  Errors:
+ * GNMR_ERR_INVALID_ARG, GNMR_ERR_STATE, GNMR_ERR_CUDA. */
+gnmr_status gnmr_finish(gnmr_handle *h, const double *d_sumsq, void *stream, uint8_t *d_mask,
+                        const gnmr_stats *stats);
+
+/* Checkpoint: copies the controller state (step counter t, and per unit A_b,
+ * k_b, Lock_b and the GNMR window Q_b) into host_buf as a self-describing
+ * blob ("GNMR", version 1, num_units, window, t, then the per-unit records and
+ * windows; little-endian).  *state_bytes (if not NULL) receives the blob size;
+ * with host_buf == NULL nothing else happens.  Waits for `stream` (work
+ * enqueued on it before the call is included), then returns.  Errors:
+ * GNMR_ERR_INVALID_ARG (buf_bytes too small), GNMR_ERR_STATE, GNMR_ERR_CUDA. */
+gnmr_status gnmr_get_state(gnmr_handle *h, void *stream, void *host_buf, int64_t buf_bytes,
+                           int64_t *state_bytes);
+
+/* Resume: loads a blob written by gnmr_get_state for the same num_units and
+ * window into the handle (on `stream`, waited for before returning), so the
+ * following steps continue the saved trace exactly.  Errors:
+ * GNMR_ERR_INVALID_ARG (NULL, short, foreign or mismatched blob, or a record
+ * out of range; the handle is unchanged), GNMR_ERR_STATE, GNMR_ERR_CUDA. */
+gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, int64_t buf_bytes);
+
 /* Overrides alpha_t and beta_t for the following steps ("scheduled
  * relaxation", Sec. 3.4).  NaN for either value returns it to the two-stage
  * schedule.  Other values must be finite and > 0 (else

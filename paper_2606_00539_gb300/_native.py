@@ -91,6 +91,10 @@ PROTOTYPES = {
                                            _P, _P, _P, _P, _P]),
     "gnmr_unit_norms_static": (ctypes.c_int, [_P, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                               _P, _P, _P, _P]),
+    "gnmr_step_partials": (ctypes.c_int, [_P, _P, ctypes.c_int64, _P, _P]),
+    "gnmr_finish": (ctypes.c_int, [_P, _P, _P, _P, ctypes.POINTER(gnmr_stats)]),
+    "gnmr_get_state": (ctypes.c_int, [_P, _P, _P, ctypes.c_int64, ctypes.POINTER(ctypes.c_int64)]),
+    "gnmr_set_state": (ctypes.c_int, [_P, _P, _P, ctypes.c_int64]),
 }
 
 _lib = None
@@ -146,6 +150,32 @@ def gnmr_step(handle: int, d_arena: int, arena_elems: int, stream: int, d_mask: 
     st = load().gnmr_step(handle, d_arena, int(arena_elems), stream, d_mask,
                           ctypes.byref(stats) if stats is not None else None)
     _check(st, handle)
+
+
+def gnmr_step_partials(handle: int, d_arena: int, arena_elems: int, stream: int, d_sumsq: int) -> None:
+    _check(load().gnmr_step_partials(handle, d_arena, int(arena_elems), stream, d_sumsq), handle)
+
+
+def gnmr_finish(handle: int, d_sumsq: int, stream: int, d_mask: int,
+                stats: gnmr_stats | None = None) -> None:
+    st = load().gnmr_finish(handle, d_sumsq, stream, d_mask,
+                            ctypes.byref(stats) if stats is not None else None)
+    _check(st, handle)
+
+
+def gnmr_get_state(handle: int, stream: int = 0) -> bytes:
+    """Returns the controller state blob."""
+    lib = load()
+    size = ctypes.c_int64(0)
+    _check(lib.gnmr_get_state(handle, stream, None, 0, ctypes.byref(size)), handle)
+    buf = ctypes.create_string_buffer(size.value)
+    _check(lib.gnmr_get_state(handle, stream, buf, size.value, ctypes.byref(size)), handle)
+    return buf.raw
+
+
+def gnmr_set_state(handle: int, blob: bytes, stream: int = 0) -> None:
+    buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+    _check(load().gnmr_set_state(handle, stream, buf, len(blob)), handle)
 
 
 def gnmr_set_thresholds(handle: int, alpha: float, beta: float) -> None:

@@ -1,6 +1,7 @@
 // Host side of the libgnmr C ABI (include/gnmr.h): argument and layout
 // validation, the work plan, the single device allocation that holds all
 // library-owned state, and the per-step launch.
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -20,6 +21,7 @@ struct gnmr_handle {
     int32_t num_units = 0;
     int elem_bytes = 0;
     int32_t num_ctas = 0;
+    int32_t finish_ctas = 0;      // grid of the controller-only launch
     int32_t num_warps = 0;
     int64_t num_partials = 0;
     int64_t device_bytes = 0;
@@ -298,6 +300,11 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         h->elem_bytes = eb;
         h->num_warps = plan.num_warps;
         h->num_ctas = (plan.num_warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
+        {
+            const int64_t warps = (U + 31) / 32;
+            const int64_t ctas = (warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
+            h->finish_ctas = static_cast<int32_t>(std::min<int64_t>(ctas, int64_t(sms) * per_sm));
+        }
         h->num_partials = plan.num_partials;
         h->device_bytes = static_cast<int64_t>(cv.size);
         h->max_end = max_end;
@@ -354,6 +361,176 @@ gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems, 
         return fail(h, GNMR_ERR_CUDA, format("step launch: %s", cudaGetErrorString(e)));
     }
     h->steps += 1;
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_step_partials(gnmr_handle *h, const void *d_arena, int64_t arena_elems, void *stream,
+                               double *d_sumsq)
+{
+    if (!h)
+        return GNMR_ERR_INVALID_ARG;
+    if (h->broken)
+        return fail(h, GNMR_ERR_STATE, "an earlier step failed in CUDA; destroy the handle");
+    if (!d_sumsq)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_sumsq must not be NULL");
+    if (arena_elems < 0)
+        return fail(h, GNMR_ERR_INVALID_ARG, "arena_elems must be >= 0");
+    if (!d_arena && h->max_end > 0)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_arena is NULL but units are not empty");
+    if (reinterpret_cast<uintptr_t>(d_arena) % static_cast<uintptr_t>(h->elem_bytes) != 0)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_arena is not aligned to the element size");
+    if (arena_elems < h->max_end)
+        return fail(h, GNMR_ERR_LAYOUT,
+                    format("arena holds %lld elements but the layout needs %lld",
+                           (long long)arena_elems, (long long)h->max_end));
+    DeviceScope scope(h->cfg.device);
+    if (scope.status() != cudaSuccess)
+        return fail(h, GNMR_ERR_CUDA, format("cudaSetDevice: %s", cudaGetErrorString(scope.status())));
+    gnmr::StepParams p = h->params;
+    p.arena = d_arena;
+    p.out_sumsq = d_sumsq;
+    const cudaError_t e = gnmr::launch_step(p, h->cfg.dtype, h->num_ctas, static_cast<cudaStream_t>(stream),
+                                            gnmr::kStepPartials);
+    if (e != cudaSuccess) {
+        h->broken = true;
+        return fail(h, GNMR_ERR_CUDA, format("partials launch: %s", cudaGetErrorString(e)));
+    }
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_finish(gnmr_handle *h, const double *d_sumsq, void *stream, uint8_t *d_mask,
+                        const gnmr_stats *stats)
+{
+    if (!h)
+        return GNMR_ERR_INVALID_ARG;
+    if (h->broken)
+        return fail(h, GNMR_ERR_STATE, "an earlier step failed in CUDA; destroy the handle");
+    if (!d_sumsq || !d_mask)
+        return fail(h, GNMR_ERR_INVALID_ARG, "d_sumsq and d_mask must not be NULL");
+    DeviceScope scope(h->cfg.device);
+    if (scope.status() != cudaSuccess)
+        return fail(h, GNMR_ERR_CUDA, format("cudaSetDevice: %s", cudaGetErrorString(scope.status())));
+    gnmr::StepParams p = h->params;
+    p.in_sumsq = d_sumsq;
+    p.mask = d_mask;
+    if (stats) {
+        p.out_norm = stats->norm;
+        p.out_gnmr = stats->gnmr;
+        p.out_dgnmr = stats->dgnmr;
+        p.out_risk = stats->risk;
+        p.out_lock = stats->lock;
+        p.out_counts = stats->counts;
+    }
+    p.alpha_override = h->alpha_override;
+    p.beta_override = h->beta_override;
+    const cudaError_t e = gnmr::launch_step(p, h->cfg.dtype, h->finish_ctas, static_cast<cudaStream_t>(stream),
+                                            gnmr::kStepFinish);
+    if (e != cudaSuccess) {
+        h->broken = true;
+        return fail(h, GNMR_ERR_CUDA, format("finish launch: %s", cudaGetErrorString(e)));
+    }
+    h->steps += 1;
+    return GNMR_OK;
+}
+
+static int64_t state_blob_bytes(const gnmr_handle *h)
+{
+    return static_cast<int64_t>(sizeof(gnmr::StateHeader)) +
+           static_cast<int64_t>(sizeof(gnmr::UnitState)) * h->num_units +
+           static_cast<int64_t>(sizeof(double)) * h->num_units * h->cfg.window;
+}
+
+gnmr_status gnmr_get_state(gnmr_handle *h, void *stream, void *host_buf, int64_t buf_bytes,
+                           int64_t *state_bytes)
+{
+    if (!h)
+        return GNMR_ERR_INVALID_ARG;
+    const int64_t need = state_blob_bytes(h);
+    if (state_bytes)
+        *state_bytes = need;
+    if (!host_buf)
+        return GNMR_OK;
+    if (buf_bytes < need)
+        return fail(h, GNMR_ERR_INVALID_ARG, format("state needs %lld bytes", (long long)need));
+    if (h->broken)
+        return fail(h, GNMR_ERR_STATE, "an earlier step failed in CUDA; destroy the handle");
+    DeviceScope scope(h->cfg.device);
+    if (scope.status() != cudaSuccess)
+        return fail(h, GNMR_ERR_CUDA, format("cudaSetDevice: %s", cudaGetErrorString(scope.status())));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    char *out = static_cast<char *>(host_buf);
+    gnmr::Control ctl{};
+    const size_t units_bytes = sizeof(gnmr::UnitState) * h->num_units;
+    const size_t queue_bytes = sizeof(double) * h->num_units * h->cfg.window;
+    cudaError_t e = cudaMemcpyAsync(&ctl, h->params.ctl, sizeof ctl, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(out + sizeof(gnmr::StateHeader), h->params.state, units_bytes,
+                            cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(out + sizeof(gnmr::StateHeader) + units_bytes, h->params.queue, queue_bytes,
+                            cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+        e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess)
+        return fail(h, GNMR_ERR_CUDA, format("state copy: %s", cudaGetErrorString(e)));
+    gnmr::StateHeader hdr{};
+    std::memcpy(hdr.magic, "GNMR", 4);
+    hdr.version = 1;
+    hdr.num_units = h->num_units;
+    hdr.window = h->cfg.window;
+    hdr.steps = ctl.steps;
+    std::memcpy(out, &hdr, sizeof hdr);
+    return GNMR_OK;
+}
+
+gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, int64_t buf_bytes)
+{
+    if (!h || !host_buf)
+        return h ? fail(h, GNMR_ERR_INVALID_ARG, "host_buf must not be NULL") : GNMR_ERR_INVALID_ARG;
+    const int64_t need = state_blob_bytes(h);
+    if (buf_bytes < need)
+        return fail(h, GNMR_ERR_INVALID_ARG, format("state needs %lld bytes", (long long)need));
+    gnmr::StateHeader hdr{};
+    std::memcpy(&hdr, host_buf, sizeof hdr);
+    if (std::memcmp(hdr.magic, "GNMR", 4) != 0 || hdr.version != 1)
+        return fail(h, GNMR_ERR_INVALID_ARG, "not a GNMR state blob (magic/version)");
+    if (hdr.num_units != h->num_units || hdr.window != h->cfg.window || hdr.steps < 0)
+        return fail(h, GNMR_ERR_INVALID_ARG,
+                    format("state is for %d units / window %d; handle has %d / %d", hdr.num_units,
+                           hdr.window, h->num_units, h->cfg.window));
+    const char *in = static_cast<const char *>(host_buf);
+    const size_t units_bytes = sizeof(gnmr::UnitState) * h->num_units;
+    const size_t queue_bytes = sizeof(double) * h->num_units * h->cfg.window;
+    for (int32_t b = 0; b < h->num_units; ++b) {
+        gnmr::UnitState u;
+        std::memcpy(&u, in + sizeof hdr + sizeof u * b, sizeof u);
+        if (u.count < 0 || u.fill < 0 || u.fill > h->cfg.window || u.head < 0 || u.head >= h->cfg.window ||
+            u.lock < 0 || u.lock > h->cfg.lock_len)
+            return fail(h, GNMR_ERR_INVALID_ARG, format("state of unit %d is out of range", b));
+    }
+    if (h->broken)
+        return fail(h, GNMR_ERR_STATE, "an earlier step failed in CUDA; destroy the handle");
+    DeviceScope scope(h->cfg.device);
+    if (scope.status() != cudaSuccess)
+        return fail(h, GNMR_ERR_CUDA, format("cudaSetDevice: %s", cudaGetErrorString(scope.status())));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    gnmr::Control ctl{};
+    ctl.steps = hdr.steps;
+    cudaError_t e = cudaMemcpyAsync(h->params.state, in + sizeof hdr, units_bytes, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->params.queue, in + sizeof hdr + units_bytes, queue_bytes,
+                            cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->params.ctl, &ctl, sizeof ctl, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(h->params.unit_ticket, 0, sizeof(uint32_t) * h->num_units, st);
+    if (e == cudaSuccess)
+        e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        h->broken = true;
+        return fail(h, GNMR_ERR_CUDA, format("state copy: %s", cudaGetErrorString(e)));
+    }
+    h->steps = hdr.steps;
     return GNMR_OK;
 }
 

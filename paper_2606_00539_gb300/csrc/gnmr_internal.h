@@ -48,6 +48,17 @@ struct Control {
     int64_t steps;        // completed steps (t of the last step)
 };
 
+// Checkpoint blob: this header, then UnitState[num_units], then the GNMR ring
+// buffers double[num_units * window] (little-endian, as on the device).
+struct StateHeader {
+    char magic[4];        // "GNMR"
+    uint32_t version;     // 1
+    int32_t num_units;
+    int32_t window;
+    int64_t steps;
+    int64_t reserved;
+};
+
 struct StepParams {
     const void *arena;
     const int64_t *offset;       // [U]
@@ -67,6 +78,8 @@ struct StepParams {
     uint8_t *mask;               // [U], caller
     double *out_norm, *out_gnmr, *out_dgnmr, *out_risk;  // caller, optional
     int32_t *out_lock, *out_counts;                       // caller, optional
+    double *out_sumsq;                                    // kStepPartials output [U]
+    const double *in_sumsq;                               // kStepFinish input [U]
     int32_t num_units;
     int32_t num_warps;
     int32_t window;
@@ -78,8 +91,15 @@ struct StepParams {
     double alpha_override, beta_override;  // NaN = two-stage schedule
 };
 
-// Enqueues one step; returns the launch status.
-cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream);
+// Step kernel modes: the full step, its gradient half (per-unit sums of
+// squares only) and its controller half (Algorithms 1-2 on given sums).
+constexpr int kStepFull = 0;
+constexpr int kStepPartials = 1;
+constexpr int kStepFinish = 2;
+
+// Enqueues one launch of the step kernel in `mode`; returns the launch status.
+cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream,
+                        int mode = kStepFull);
 
 // Resident CTAs per SM of the step kernel for `dtype`.
 cudaError_t step_occupancy(int dtype, int *ctas_per_sm);

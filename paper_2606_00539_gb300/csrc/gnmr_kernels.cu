@@ -23,6 +23,10 @@
 // Algorithm 2, the mask write, and the reset of the counters for the next
 // launch.  No CTA ever waits for another: the tickets decide who continues,
 // so the kernel cannot hang whatever the grid size or residency.
+//
+// The same kernel also runs either half of a sharded step: phase 1 alone
+// (per-unit sums of squares of a shard) or phases 2-3 alone on sums that the
+// caller has added up across shards.
 #include <cstdint>
 
 #include <cuda_runtime.h>
@@ -473,7 +477,11 @@ __device__ void select_and_commit(const StepParams &p, uint32_t *hist, uint32_t 
     }
 }
 
-template <int DT>
+// MODE kStepFull: the whole step.  kStepPartials: phase 1 only, each unit's
+// sum of squares written to out_sumsq (the first half of a sharded step).
+// kStepFinish: no gradient read; phases 2-3 on the sums in in_sumsq (the
+// second half, after the caller has reduced the shards' sums).
+template <int DT, int MODE>
 __global__ void __launch_bounds__(kThreads, kMinCtasPerSm)
 gnmr_step_kernel(const __grid_constant__ StepParams p)
 {
@@ -483,7 +491,18 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     const int lane = threadIdx.x & 31;
     const int warp = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
 
-    if (warp < p.num_warps) {
+    if (MODE == kStepFinish) {
+        const int64_t t = __ldcg(&p.ctl->steps) + 1;
+        const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
+        const double beta = pick_threshold(p.beta_override, t, p.warmup_steps, p.beta_init, p.beta_main);
+        const int64_t warps = static_cast<int64_t>(gridDim.x) * kWarpsPerCta;
+        for (int64_t b0 = static_cast<int64_t>(warp) * 32; b0 < p.num_units; b0 += warps * 32) {
+            const int64_t b = b0 + lane;
+            const bool active = b < p.num_units;
+            const double s = active ? p.in_sumsq[b] : 0.0;
+            unit_epilogue(p, active, active ? static_cast<int32_t>(b) : 0, s, alpha, beta);
+        }
+    } else if (warp < p.num_warps) {
         // t, alpha_t and beta_t are fixed for the whole step.
         const int64_t t = __ldcg(&p.ctl->steps) + 1;
         const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
@@ -510,21 +529,28 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
             if (suspect)
                 s = warp_segment_sumsq_f64<DT>(seg, n, lane);
             if (parts == 1 || combine_parts(p, b, parts, warp, s, lane)) {
-                if (lane == npend) {
-                    pend_b = b;
-                    pend_s = s;
-                }
-                if (++npend == 32) {
-                    unit_epilogue(p, true, pend_b, pend_s, alpha, beta);
-                    npend = 0;
+                if (MODE == kStepPartials) {
+                    if (lane == 0)
+                        p.out_sumsq[b] = s;
+                } else {
+                    if (lane == npend) {
+                        pend_b = b;
+                        pend_s = s;
+                    }
+                    if (++npend == 32) {
+                        unit_epilogue(p, true, pend_b, pend_s, alpha, beta);
+                        npend = 0;
+                    }
                 }
             }
             ++b;
             pos = 0;
         }
-        if (npend > 0)
+        if (MODE != kStepPartials && npend > 0)
             unit_epilogue(p, lane < npend, pend_b, pend_s, alpha, beta);
     }
+    if (MODE == kStepPartials)
+        return;
 
     // Grid completion: the last CTA through runs the selection.
     __threadfence();
@@ -538,22 +564,34 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     }
 }
 
-}  // namespace
-
-cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream)
+template <int MODE>
+cudaError_t launch_mode(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream)
 {
     if (dtype == 1)
-        gnmr_step_kernel<1><<<num_ctas, kThreads, 0, stream>>>(p);
+        gnmr_step_kernel<1, MODE><<<num_ctas, kThreads, 0, stream>>>(p);
     else
-        gnmr_step_kernel<0><<<num_ctas, kThreads, 0, stream>>>(p);
+        gnmr_step_kernel<0, MODE><<<num_ctas, kThreads, 0, stream>>>(p);
     return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream, int mode)
+{
+    if (mode == kStepPartials)
+        return launch_mode<kStepPartials>(p, dtype, num_ctas, stream);
+    if (mode == kStepFinish)
+        return launch_mode<kStepFinish>(p, 0, num_ctas, stream);
+    return launch_mode<kStepFull>(p, dtype, num_ctas, stream);
 }
 
 cudaError_t step_occupancy(int dtype, int *ctas_per_sm)
 {
     if (dtype == 1)
-        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<1>, kThreads, 0);
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<0>, kThreads, 0);
+        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<1, kStepFull>,
+                                                             kThreads, 0);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<0, kStepFull>,
+                                                         kThreads, 0);
 }
 
 }  // namespace gnmr

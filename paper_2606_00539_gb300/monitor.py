@@ -2,7 +2,6 @@
 the CUDA stream; every step of the monitor runs in libgnmr's kernel."""
 from __future__ import annotations
 
-import ctypes
 import math
 
 import numpy as np
@@ -116,6 +115,61 @@ class Monitor:
         if numel is not None and t.numel() < numel:
             raise ValueError(f"{name} must hold at least {numel} elements")
 
+    def _stats_struct(self, stats):
+        torch = _torch()
+        if stats is None:
+            return None
+        st = N.gnmr_stats()
+        for key, dt, n in (("norm", torch.float64, self.num_units),
+                           ("gnmr", torch.float64, self.num_units),
+                           ("dgnmr", torch.float64, self.num_units),
+                           ("risk", torch.float64, self.num_units),
+                           ("lock", torch.int32, self.num_units),
+                           ("counts", torch.int32, 2)):
+            if stats.get(key) is not None:
+                self._check_tensor(stats[key], key, dt, n)
+                setattr(st, key, stats[key].data_ptr())
+        return st
+
+    def _stream_handle(self, stream, device):
+        torch = _torch()
+        if stream is None:
+            stream = torch.cuda.current_stream(device)
+        return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+    def step_partials(self, arena, sumsq=None, stream=None):
+        """First half of a sharded step: per-unit sums of squares of this
+        rank's local arena (fp64 tensor [U]); no controller state changes."""
+        torch = _torch()
+        want = torch.bfloat16 if self.dtype == N.GNMR_DTYPE_BF16 else torch.float32
+        self._check_tensor(arena, "arena", want)
+        if sumsq is None:
+            sumsq = torch.empty(self.num_units, dtype=torch.float64, device=arena.device)
+        self._check_tensor(sumsq, "sumsq", torch.float64, self.num_units)
+        N.gnmr_step_partials(self._h, arena.data_ptr(), arena.numel(),
+                             self._stream_handle(stream, arena.device), sumsq.data_ptr())
+        return sumsq
+
+    def finish(self, sumsq, mask=None, stats: dict | None = None, stream=None):
+        """Second half: one controller step on summed sums of squares."""
+        torch = _torch()
+        self._check_tensor(sumsq, "sumsq", torch.float64, self.num_units)
+        if mask is None:
+            mask = torch.empty(self.num_units, dtype=torch.uint8, device=sumsq.device)
+        self._check_tensor(mask, "mask", torch.uint8, self.num_units)
+        N.gnmr_finish(self._h, sumsq.data_ptr(), self._stream_handle(stream, sumsq.device),
+                      mask.data_ptr(), self._stats_struct(stats))
+        return mask
+
+    def get_state(self, stream=None) -> bytes:
+        """Checkpoint blob of the controller state (waits for the stream)."""
+        torch = _torch()
+        return N.gnmr_get_state(self._h, self._stream_handle(stream, torch.device("cuda", self.device_index)))
+
+    def set_state(self, blob: bytes, stream=None) -> None:
+        torch = _torch()
+        N.gnmr_set_state(self._h, blob, self._stream_handle(stream, torch.device("cuda", self.device_index)))
+
     def step(self, arena, mask=None, stats: dict | None = None, stream=None):
         """Enqueues one GNMR step on `stream` (default: torch's current
         stream) and returns the uint8 mask tensor (1 = recovery path)."""
@@ -125,20 +179,6 @@ class Monitor:
         if mask is None:
             mask = torch.empty(self.num_units, dtype=torch.uint8, device=arena.device)
         self._check_tensor(mask, "mask", torch.uint8, self.num_units)
-        st = None
-        if stats is not None:
-            st = N.gnmr_stats()
-            for key, dt, n in (("norm", torch.float64, self.num_units),
-                               ("gnmr", torch.float64, self.num_units),
-                               ("dgnmr", torch.float64, self.num_units),
-                               ("risk", torch.float64, self.num_units),
-                               ("lock", torch.int32, self.num_units),
-                               ("counts", torch.int32, 2)):
-                if stats.get(key) is not None:
-                    self._check_tensor(stats[key], key, dt, n)
-                    setattr(st, key, stats[key].data_ptr())
-        if stream is None:
-            stream = torch.cuda.current_stream(arena.device)
-        s = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
-        N.gnmr_step(self._h, arena.data_ptr(), arena.numel(), s, mask.data_ptr(), st)
+        N.gnmr_step(self._h, arena.data_ptr(), arena.numel(), self._stream_handle(stream, arena.device),
+                    mask.data_ptr(), self._stats_struct(stats))
         return mask
