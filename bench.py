@@ -42,6 +42,8 @@ def parse_args(argv=None):
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["gnmr", "reference"], default="gnmr")
     p.add_argument("--workload", default="llama2-13b")
+    p.add_argument("--group", default="tensor", choices=["tensor", "block", "expert"],
+                   help="unit granularity: one per tensor, per transformer block, per MoE expert")
     p.add_argument("--shrink", type=int, default=1,
                    help="divide matrix dims (small case for profiler captures)")
     p.add_argument("--arenas", type=int, default=2, help="distinct step arenas cycled")
@@ -285,7 +287,7 @@ def run_gnmr(args):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
 
-    w = workloads.make(args.workload, shrink=args.shrink, seed=rank)
+    w = workloads.make(args.workload, shrink=args.shrink, seed=rank, group=args.group)
     filler = workloads.Filler(w, dev)
     n_arenas = max(1, args.arenas)
     arenas = []
@@ -402,7 +404,8 @@ def run_gnmr(args):
             "pct_hbm_peak": round(100 * value / world / peak, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": w.dtype, "data": "synthetic",
-            "config": {"workload": f"{w.name} ({w.num_units} units, {w.grad_elems} {w.dtype} "
+            "config": {"workload": f"{w.name} ({w.num_units} units, {w.num_segments} tensors, "
+                                   f"{w.grad_elems} {w.dtype} "
                                    f"elements{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
                        "bytes_per_step": w.grad_bytes, "arenas_cycled": n_arenas,
                        "l2": ("L2 flushed before every step (512 MB write)" if args.flush_l2

@@ -56,8 +56,8 @@ typedef enum gnmr_dtype {
  * with the values listed per field. */
 typedef struct gnmr_config {
     int32_t num_units;            /* |B|, monitored units, >= 1 (no default) */
-    const int64_t *offsets;       /* host [num_units]: first element of unit b in the arena, >= 0 */
-    const int64_t *lengths;       /* host [num_units]: elements of unit b, >= 0 (0 = empty unit, norm 0) */
+    const int64_t *offsets;       /* host [num_units] (or [num_segments]): first element in the arena, >= 0 */
+    const int64_t *lengths;       /* host, same count: elements, >= 0 (0 = empty, norm 0) */
     const uint8_t *recoverable;   /* host [num_units], nonzero = b in B_rec; NULL = every unit recoverable */
     int32_t dtype;                /* gnmr_dtype of the arena; default GNMR_DTYPE_BF16 */
     int32_t window;               /* delta, Delta-GNMR window, >= 1; default 8 */
@@ -70,6 +70,15 @@ typedef struct gnmr_config {
     int64_t warmup_steps;         /* length of the first threshold stage, >= 0; default 0 */
     double eps;                   /* epsilon of Algorithm 1, >= 0; default 1e-8 */
     int32_t device;               /* CUDA device ordinal; default 0 */
+    /* Multi-segment units (Sec. 3.4: a whole transformer block as one
+     * recoverable unit, all its operators sharing one decision).  0 (default):
+     * unit b is the single segment offsets[b], lengths[b].  > 0: offsets and
+     * lengths describe num_segments segments and segment_unit[s] in
+     * [0, num_units) names the unit each belongs to; n_b is the L2 norm over
+     * all of b's segments (a unit with none has n_b = 0).  Segments may come in
+     * any order; a unit's segments are summed in the order given. */
+    int32_t num_segments;
+    const int32_t *segment_unit;  /* host [num_segments] when num_segments > 0, else ignored */
 } gnmr_config;
 
 /* Optional per-step statistics: caller-owned DEVICE buffers.  Any pointer

@@ -55,6 +55,9 @@ def _load():
     P = ctypes.c_void_p
     lib.oracle_unit_norms.argtypes = [P, ctypes.c_int, P, P, ctypes.c_int32, P]
     lib.oracle_unit_norms.restype = ctypes.c_int
+    lib.oracle_unit_norms_segmented.argtypes = [P, ctypes.c_int, P, P, P, ctypes.c_int64,
+                                                ctypes.c_int32, P]
+    lib.oracle_unit_norms_segmented.restype = ctypes.c_int
     lib.oracle_ctl_create.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                       ctypes.c_int32, ctypes.c_int64, ctypes.c_double,
                                       ctypes.c_double, ctypes.c_double, ctypes.c_double,
@@ -126,6 +129,48 @@ def unit_norms_threaded(arena: np.ndarray, offsets, lengths, threads: int) -> np
 
     with ThreadPoolExecutor(max_workers=len(bounds) - 1) as ex:
         list(ex.map(run, range(len(bounds) - 1)))
+    return out
+
+
+def unit_norms_segmented(arena: np.ndarray, offsets, lengths, segment_unit, num_units: int,
+                         threads: int = 1) -> np.ndarray:
+    """n_b over units made of several segments (Eq. local_gradient for a
+    whole block, Sec. 3.4).  ``offsets``/``lengths``/``segment_unit`` describe
+    the segments; the units are split over ``threads`` host threads, each
+    running the same plain C loop over its units' segments."""
+    arena = np.ascontiguousarray(arena).reshape(-1)
+    off = np.ascontiguousarray(offsets, dtype=np.int64)
+    ln = np.ascontiguousarray(lengths, dtype=np.int64)
+    su = np.ascontiguousarray(segment_unit, dtype=np.int32)
+    if not (off.shape == ln.shape == su.shape):
+        raise ValueError("segment arrays differ in length")
+    if len(off) and (np.any(off < 0) or np.any(ln < 0) or np.max(off + ln) > arena.size
+                     or su.min() < 0 or su.max() >= num_units):
+        raise ValueError("segment layout exceeds the arena or the unit range")
+    lib = _load()
+    dt = _arena_dtype(arena)
+    out = np.zeros(num_units, dtype=np.float64)
+    threads = max(1, min(int(threads), num_units))
+    bounds = np.linspace(0, num_units, threads + 1).astype(int)
+
+    def run(i):
+        a, b = bounds[i], bounds[i + 1]
+        sel = np.nonzero((su >= a) & (su < b))[0]
+        part = np.empty(b - a, dtype=np.float64)
+        o = np.ascontiguousarray(off[sel])       # kept alive across the C call
+        n = np.ascontiguousarray(ln[sel])
+        u = np.ascontiguousarray(su[sel] - a, dtype=np.int32)
+        rc = lib.oracle_unit_norms_segmented(_ptr(arena), dt, _ptr(o), _ptr(n), _ptr(u), len(sel),
+                                             b - a, _ptr(part))
+        if rc != 0:
+            raise RuntimeError("oracle_unit_norms_segmented failed")
+        out[a:b] = part
+
+    if threads == 1:
+        run(0)
+    else:
+        with ThreadPoolExecutor(max_workers=threads) as ex:
+            list(ex.map(run, range(threads)))
     return out
 
 

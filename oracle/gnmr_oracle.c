@@ -73,6 +73,43 @@ int oracle_unit_norms(const void *arena, int dtype, const int64_t *offsets,
     return 0;
 }
 
+/* Eq. local_gradient for units made of several segments (Sec. 3.4: a whole
+ * transformer block as one unit): n_b = sqrt of the sum of squares over
+ * every element of every segment of b, one running sum per unit, segments in
+ * the order given.  A unit with no segment has n_b = 0. */
+int oracle_unit_norms_segmented(const void *arena, int dtype, const int64_t *offsets,
+                                const int64_t *lengths, const int32_t *segment_unit,
+                                int64_t num_segments, int32_t num_units, double *norms)
+{
+    if (dtype != ORACLE_DTYPE_F32 && dtype != ORACLE_DTYPE_BF16)
+        return 1;
+    for (int32_t b = 0; b < num_units; ++b)
+        norms[b] = 0.0;                      /* running sums of squares */
+    for (int64_t g = 0; g < num_segments; ++g) {
+        const int32_t b = segment_unit[g];
+        if (b < 0 || b >= num_units)
+            return 2;
+        double sum = norms[b];
+        if (dtype == ORACLE_DTYPE_F32) {
+            const float *x = (const float *)arena + offsets[g];
+            for (int64_t i = 0; i < lengths[g]; ++i) {
+                double v = (double)x[i];
+                sum += v * v;
+            }
+        } else {
+            const uint16_t *x = (const uint16_t *)arena + offsets[g];
+            for (int64_t i = 0; i < lengths[g]; ++i) {
+                double v = bf16_to_double(x[i]);
+                sum += v * v;
+            }
+        }
+        norms[b] = sum;
+    }
+    for (int32_t b = 0; b < num_units; ++b)
+        norms[b] = sqrt(norms[b]);
+    return 0;
+}
+
 /* Per-unit controller state: A_b (historical mean), Q_b (the last <= delta
  * GNMR values, oldest first), k_b (observation count), Lock_b. */
 typedef struct {

@@ -41,6 +41,8 @@ class gnmr_config(ctypes.Structure):
         ("warmup_steps", ctypes.c_int64),
         ("eps", ctypes.c_double),
         ("device", ctypes.c_int32),
+        ("num_segments", ctypes.c_int32),
+        ("segment_unit", _P),
     ]
 
 

@@ -23,6 +23,7 @@ struct gnmr_handle {
     int32_t num_ctas = 0;
     int32_t finish_ctas = 0;      // grid of the controller-only launch
     int32_t num_warps = 0;
+    int64_t num_segments = 0;
     int64_t num_partials = 0;
     int64_t device_bytes = 0;
     int64_t max_end = 0;
@@ -147,13 +148,18 @@ gnmr_status gnmr_plan_partition(int32_t num_units, const int64_t *lengths, int32
         return GNMR_ERR_INVALID_ARG;
     gnmr::Plan plan;
     try {
-        if (!gnmr::plan_partition(num_units, lengths, dtype == GNMR_DTYPE_BF16 ? 2 : 4, max_warps, plan))
+        std::vector<int32_t> ident(num_units);
+        for (int32_t u = 0; u < num_units; ++u)
+            ident[u] = u;
+        if (!gnmr::plan_partition(num_units, lengths, ident.data(), num_units,
+                                  dtype == GNMR_DTYPE_BF16 ? 2 : 4, max_warps, plan))
             return GNMR_ERR_INVALID_ARG;
     } catch (const std::bad_alloc &) {
         return GNMR_ERR_OOM;
     }
     *num_warps = plan.num_warps;
-    std::memcpy(run_unit, plan.run_unit.data(), sizeof(int32_t) * (plan.num_warps + 1));
+    for (int32_t w = 0; w <= plan.num_warps; ++w)
+        run_unit[w] = static_cast<int32_t>(plan.run_seg[w]);
     std::memcpy(run_pos, plan.run_pos.data(), sizeof(int64_t) * (plan.num_warps + 1));
     std::memcpy(first_warp, plan.first_warp.data(), sizeof(int32_t) * num_units);
     std::memcpy(num_parts, plan.num_parts.data(), sizeof(int32_t) * num_units);
@@ -182,15 +188,22 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         return fail_create(GNMR_ERR_INVALID_ARG, "thresholds alpha/beta must be finite and > 0");
     if (!std::isfinite(c.eps) || c.eps < 0.0)
         return fail_create(GNMR_ERR_INVALID_ARG, "eps must be finite and >= 0");
+    if (c.num_segments < 0 || (c.num_segments > 0 && !c.segment_unit))
+        return fail_create(GNMR_ERR_INVALID_ARG, "num_segments must be >= 0, with segment_unit when > 0");
     const int eb = c.dtype == GNMR_DTYPE_BF16 ? 2 : 4;
     const int64_t limit = std::numeric_limits<int64_t>::max() / 8;
+    const int64_t S_in = c.num_segments > 0 ? c.num_segments : c.num_units;
     int64_t max_end = 0;
-    for (int32_t b = 0; b < c.num_units; ++b) {
-        const int64_t o = c.offsets[b], l = c.lengths[b];
+    for (int64_t g = 0; g < S_in; ++g) {
+        const int64_t o = c.offsets[g], l = c.lengths[g];
         if (o < 0 || l < 0 || o > limit - l)
             return fail_create(GNMR_ERR_INVALID_ARG,
-                               format("unit %d: offset %lld / length %lld out of range", b,
+                               format("%s %lld: offset %lld / length %lld out of range",
+                                      c.num_segments > 0 ? "segment" : "unit", (long long)g,
                                       (long long)o, (long long)l));
+        if (c.num_segments > 0 && (c.segment_unit[g] < 0 || c.segment_unit[g] >= c.num_units))
+            return fail_create(GNMR_ERR_INVALID_ARG,
+                               format("segment %lld: unit %d out of range", (long long)g, c.segment_unit[g]));
         if (l > 0 && o + l > max_end)
             max_end = o + l;
     }
@@ -216,17 +229,54 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         return fail_create(GNMR_ERR_OOM, "host allocation failed");
     const int64_t U = c.num_units;
     try {
+        // Segments grouped by unit (stable: a unit keeps its segments' order);
+        // a unit without segments gets one empty segment.
+        std::vector<int64_t> seg_off, seg_len;
+        std::vector<int32_t> seg_unit;
+        if (c.num_segments > 0) {
+            std::vector<int64_t> order(S_in);
+            for (int64_t g = 0; g < S_in; ++g)
+                order[g] = g;
+            std::stable_sort(order.begin(), order.end(), [&](int64_t a, int64_t b) {
+                return c.segment_unit[a] < c.segment_unit[b];
+            });
+            seg_off.reserve(S_in + U);
+            size_t k = 0;
+            for (int32_t u = 0; u < c.num_units; ++u) {
+                const size_t before = seg_off.size();
+                while (k < order.size() && c.segment_unit[order[k]] == u) {
+                    seg_off.push_back(c.offsets[order[k]]);
+                    seg_len.push_back(c.lengths[order[k]]);
+                    seg_unit.push_back(u);
+                    ++k;
+                }
+                if (seg_off.size() == before) {
+                    seg_off.push_back(0);
+                    seg_len.push_back(0);
+                    seg_unit.push_back(u);
+                }
+            }
+        } else {
+            seg_off.assign(c.offsets, c.offsets + U);
+            seg_len.assign(c.lengths, c.lengths + U);
+            seg_unit.resize(U);
+            for (int32_t u = 0; u < c.num_units; ++u)
+                seg_unit[u] = u;
+        }
+        const int64_t S = static_cast<int64_t>(seg_off.size());
         gnmr::Plan plan;
-        if (!gnmr::plan_partition(c.num_units, c.lengths, eb, sms * per_sm * gnmr::kWarpsPerCta, plan)) {
+        if (!gnmr::plan_partition(S, seg_len.data(), seg_unit.data(), c.num_units, eb,
+                                  sms * per_sm * gnmr::kWarpsPerCta, plan)) {
             delete h;
             return fail_create(GNMR_ERR_INVALID_ARG, "work partition failed (sizes out of range)");
         }
         const int64_t W = plan.num_warps;
         Carver cv;
-        const size_t o_off = cv.take(sizeof(int64_t) * U);
-        const size_t o_len = cv.take(sizeof(int64_t) * U);
+        const size_t o_off = cv.take(sizeof(int64_t) * S);
+        const size_t o_len = cv.take(sizeof(int64_t) * S);
+        const size_t o_segu = cv.take(sizeof(int32_t) * S);
         const size_t o_rec = cv.take(U);
-        const size_t o_run_unit = cv.take(sizeof(int32_t) * (W + 1));
+        const size_t o_run_seg = cv.take(sizeof(int64_t) * (W + 1));
         const size_t o_run_pos = cv.take(sizeof(int64_t) * (W + 1));
         const size_t o_first = cv.take(sizeof(int32_t) * U);
         const size_t o_parts = cv.take(sizeof(int32_t) * U);
@@ -240,11 +290,12 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
 
         // Host image of the whole block: static tables plus zeroed state.
         std::vector<unsigned char> img(cv.size, 0);
-        std::memcpy(&img[o_off], c.offsets, sizeof(int64_t) * U);
-        std::memcpy(&img[o_len], c.lengths, sizeof(int64_t) * U);
+        std::memcpy(&img[o_off], seg_off.data(), sizeof(int64_t) * S);
+        std::memcpy(&img[o_len], seg_len.data(), sizeof(int64_t) * S);
+        std::memcpy(&img[o_segu], seg_unit.data(), sizeof(int32_t) * S);
         for (int64_t b = 0; b < U; ++b)
             img[o_rec + b] = c.recoverable ? (c.recoverable[b] != 0) : 1;
-        std::memcpy(&img[o_run_unit], plan.run_unit.data(), sizeof(int32_t) * (W + 1));
+        std::memcpy(&img[o_run_seg], plan.run_seg.data(), sizeof(int64_t) * (W + 1));
         std::memcpy(&img[o_run_pos], plan.run_pos.data(), sizeof(int64_t) * (W + 1));
         std::memcpy(&img[o_first], plan.first_warp.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_parts], plan.num_parts.data(), sizeof(int32_t) * U);
@@ -268,8 +319,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         gnmr::StepParams &p = h->params;
         p.offset = reinterpret_cast<const int64_t *>(base + o_off);
         p.length = reinterpret_cast<const int64_t *>(base + o_len);
+        p.seg_unit = reinterpret_cast<const int32_t *>(base + o_segu);
         p.recoverable = reinterpret_cast<const uint8_t *>(base + o_rec);
-        p.run_unit = reinterpret_cast<const int32_t *>(base + o_run_unit);
+        p.run_seg = reinterpret_cast<const int64_t *>(base + o_run_seg);
         p.run_pos = reinterpret_cast<const int64_t *>(base + o_run_pos);
         p.first_warp = reinterpret_cast<const int32_t *>(base + o_first);
         p.num_parts = reinterpret_cast<const int32_t *>(base + o_parts);
@@ -296,6 +348,8 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         h->cfg.offsets = nullptr;
         h->cfg.lengths = nullptr;
         h->cfg.recoverable = nullptr;
+        h->cfg.segment_unit = nullptr;
+        h->num_segments = S;
         h->num_units = c.num_units;
         h->elem_bytes = eb;
         h->num_warps = plan.num_warps;

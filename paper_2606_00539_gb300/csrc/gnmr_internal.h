@@ -61,10 +61,11 @@ struct StateHeader {
 
 struct StepParams {
     const void *arena;
-    const int64_t *offset;       // [U]
-    const int64_t *length;       // [U]
+    const int64_t *offset;       // [S] segment offsets, segments grouped by unit
+    const int64_t *length;       // [S] segment lengths
+    const int32_t *seg_unit;     // [S] unit of each segment (non-decreasing)
     const uint8_t *recoverable;  // [U]
-    const int32_t *run_unit;     // [W + 1]
+    const int64_t *run_seg;      // [W + 1] first segment of each warp's run
     const int64_t *run_pos;      // [W + 1]
     const int32_t *first_warp;   // [U]
     const int32_t *num_parts;    // [U]
@@ -111,7 +112,7 @@ void record_thread_error(const char *why);
 // Host-side work partition (gnmr_plan.cpp).
 struct Plan {
     int32_t num_warps = 0;
-    std::vector<int32_t> run_unit;    // [num_warps + 1]
+    std::vector<int64_t> run_seg;     // [num_warps + 1]
     std::vector<int64_t> run_pos;     // [num_warps + 1]
     std::vector<int32_t> first_warp;  // [U]
     std::vector<int32_t> num_parts;   // [U]
@@ -119,8 +120,9 @@ struct Plan {
     int64_t num_partials = 0;
 };
 
-// Returns false if the inputs are out of range.
-bool plan_partition(int32_t num_units, const int64_t *lengths, int elem_bytes,
-                    int32_t max_warps, Plan &out);
+// Segments must be grouped by unit (seg_unit non-decreasing, every unit
+// 0..num_units-1 present).  Returns false if the inputs are out of range.
+bool plan_partition(int64_t num_segments, const int64_t *seg_lengths, const int32_t *seg_unit,
+                    int32_t num_units, int elem_bytes, int32_t max_warps, Plan &out);
 
 }  // namespace gnmr

@@ -1,8 +1,9 @@
 // GNMR per-step monitor: one kernel launch per training step on sm_103a.
 //
 // Phase 1, every warp (the hot loop).  Each warp owns one contiguous run of
-// the unit stream planned by gnmr_plan.cpp.  For every unit segment in its
-// run it streams the gradient with 16-byte read-only loads (8 in flight per
+// the segment stream planned by gnmr_plan.cpp (a unit is one or more
+// segments of the arena).  For every segment piece in its run it streams the
+// gradient with 16-byte read-only loads (8 in flight per
 // lane, 4 KiB per warp per iteration), squares in fp32, sums blocks of 16
 // iterations in fp32 and the blocks in fp64, and all-reduces across the warp
 // with shuffles: n_b = ||g_b||_2 (Sec. 2, Eq. local_gradient).  No shared
@@ -507,9 +508,9 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
         const int64_t t = __ldcg(&p.ctl->steps) + 1;
         const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
         const double beta = pick_threshold(p.beta_override, t, p.warmup_steps, p.beta_init, p.beta_main);
-        int32_t b = p.run_unit[warp];
+        int64_t g = p.run_seg[warp];
         int64_t pos = p.run_pos[warp];
-        const int32_t b_end = p.run_unit[warp + 1];
+        const int64_t g_end = p.run_seg[warp + 1];
         const int64_t pos_end = p.run_pos[warp + 1];
         const char *arena = static_cast<const char *>(p.arena);
         // Units this warp completes wait here, lane j holding the j-th, and run
@@ -517,17 +518,12 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
         int32_t pend_b = 0;
         double pend_s = 0.0;
         int npend = 0;
-        while (b < b_end || (b == b_end && pos < pos_end)) {
-            const int64_t len = p.length[b];
+        // Segments of one unit are consecutive: their sums add up in segment
+        // order until the unit changes.
+        int32_t cur = -1;
+        double cur_s = 0.0;
+        auto complete = [&](int32_t b, double s) {
             const int32_t parts = p.num_parts[b];
-            int64_t stop = (b == b_end) ? pos_end : len;
-            stop = stop < len ? stop : len;
-            const int64_t n = stop > pos ? stop - pos : 0;
-            const char *seg = arena + (p.offset[b] + pos) * kEB;
-            bool suspect;
-            double s = warp_segment_sumsq<DT>(seg, n, lane, suspect);
-            if (suspect)
-                s = warp_segment_sumsq_f64<DT>(seg, n, lane);
             if (parts == 1 || combine_parts(p, b, parts, warp, s, lane)) {
                 if (MODE == kStepPartials) {
                     if (lane == 0)
@@ -543,9 +539,31 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
                     }
                 }
             }
-            ++b;
+        };
+        while (g < g_end || (g == g_end && pos < pos_end)) {
+            const int32_t b = p.seg_unit[g];
+            const int64_t len = p.length[g];
+            int64_t stop = (g == g_end) ? pos_end : len;
+            stop = stop < len ? stop : len;
+            const int64_t n = stop > pos ? stop - pos : 0;
+            const char *seg = arena + (p.offset[g] + pos) * kEB;
+            bool suspect;
+            double s = warp_segment_sumsq<DT>(seg, n, lane, suspect);
+            if (suspect)
+                s = warp_segment_sumsq_f64<DT>(seg, n, lane);
+            if (b != cur) {
+                if (cur >= 0)
+                    complete(cur, cur_s);
+                cur = b;
+                cur_s = s;
+            } else {
+                cur_s += s;
+            }
+            ++g;
             pos = 0;
         }
+        if (cur >= 0)
+            complete(cur, cur_s);
         if (MODE != kStepPartials && npend > 0)
             unit_epilogue(p, lane < npend, pend_b, pend_s, alpha, beta);
     }

@@ -20,7 +20,10 @@ def _torch():
 class Monitor:
     """The GNMR per-step monitor for one flat gradient arena.
 
-    offsets, lengths: per-unit element offset and length in the arena.
+    offsets, lengths: element offset and length in the arena of every unit,
+    or of every segment when segment_unit is given (segment_unit[s] = the
+    unit of segment s, for units that span several tensors, e.g. a whole
+    transformer block; num_units defaults to max(segment_unit) + 1).
     recoverable: per-unit flags (B_rec); None = every unit recoverable.
     alpha, beta: (init, main) thresholds; the init values hold for steps
     t <= warmup_steps (two-stage schedule).  A scalar means both stages.
@@ -28,16 +31,26 @@ class Monitor:
 
     def __init__(self, offsets, lengths, *, dtype="bf16", recoverable=None, window=8, max_o=4,
                  lock_len=1, alpha=(1.5, 1.1), beta=(1.5, 1.5), warmup_steps=0, eps=1e-8,
-                 device=0):
+                 device=0, segment_unit=None, num_units=None):
         self._h = None
         off = np.ascontiguousarray(offsets, dtype=np.int64)
         ln = np.ascontiguousarray(lengths, dtype=np.int64)
         if off.ndim != 1 or off.shape != ln.shape:
             raise ValueError("offsets and lengths must be 1-D arrays of equal length")
+        seg = None
+        if segment_unit is not None:
+            seg = np.ascontiguousarray(segment_unit, dtype=np.int32)
+            if seg.shape != off.shape:
+                raise ValueError("segment_unit must have one entry per segment")
+            if num_units is None:
+                num_units = int(seg.max()) + 1 if len(seg) else 0
+        elif num_units is not None and num_units != len(off):
+            raise ValueError("num_units without segment_unit must equal len(offsets)")
+        U = len(off) if num_units is None else int(num_units)
         rec = None
         if recoverable is not None:
             rec = np.ascontiguousarray(recoverable, dtype=np.uint8)
-            if rec.shape != off.shape:
+            if rec.shape != (U,):
                 raise ValueError("recoverable must have one flag per unit")
         if isinstance(alpha, (int, float)):
             alpha = (alpha, alpha)
@@ -46,7 +59,10 @@ class Monitor:
         if dtype not in _DTYPES:
             raise ValueError(f"dtype must be one of {sorted(_DTYPES)}")
         cfg = N.gnmr_config_defaults()
-        cfg.num_units = len(off)
+        cfg.num_units = U
+        if seg is not None:
+            cfg.num_segments = len(seg)
+            cfg.segment_unit = seg.ctypes.data
         cfg.offsets = off.ctypes.data
         cfg.lengths = ln.ctypes.data
         cfg.recoverable = None if rec is None else rec.ctypes.data
@@ -60,7 +76,7 @@ class Monitor:
         cfg.eps = float(eps)
         cfg.device = int(device.index if hasattr(device, "index") else device)
         self._h = N.gnmr_create(cfg)
-        self.num_units = len(off)
+        self.num_units = U
         self.dtype = cfg.dtype
         self.device_index = cfg.device
         self.arena_elems_min = int(self.info()["arena_elems_min"])

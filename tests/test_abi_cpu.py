@@ -61,6 +61,7 @@ int main(void) {
   F(gnmr_config, max_o) F(gnmr_config, lock_len) F(gnmr_config, alpha_init)
   F(gnmr_config, alpha_main) F(gnmr_config, beta_init) F(gnmr_config, beta_main)
   F(gnmr_config, warmup_steps) F(gnmr_config, eps) F(gnmr_config, device)
+  F(gnmr_config, num_segments) F(gnmr_config, segment_unit)
   F(gnmr_stats, norm) F(gnmr_stats, gnmr) F(gnmr_stats, dgnmr) F(gnmr_stats, risk)
   F(gnmr_stats, lock) F(gnmr_stats, counts)
   F(gnmr_info, num_units) F(gnmr_info, dtype) F(gnmr_info, device) F(gnmr_info, num_ctas)

@@ -56,6 +56,49 @@ def test_workload_parity(config, shrink, steps, cuda_device):
     assert sum(r.attempts for r in tr.records) < 10 * w.steps
 
 
+@pytest.mark.parametrize("config,group,shrink,steps", [
+    ("llama2-13b", "block", 16, None),     # 40 layer units of 7 tensors each
+    ("llama2-1.3b", "block", 8, 40),
+    ("moe", "expert", 16, 20),             # attention + each expert as one unit
+    ("moe", "block", 32, 20),
+])
+def test_block_level_units_parity(config, group, shrink, steps, cuda_device):
+    """Units spanning several tensors (Sec. 3.4): the unit norm covers all of
+    its tensors and the whole block shares one decision."""
+    w = workloads.make(config, shrink=shrink, steps=steps, group=group)
+    assert w.num_units < w.num_segments
+    _run_lockstep(w)
+
+
+def test_segments_in_any_order_and_units_without_segments(cuda_device):
+    import torch
+    rng = np.random.default_rng(21)
+    n = 400_000
+    off = np.array([5000, 0, 123_457, 300_001, 77, 200_000, 350_000], np.int64)
+    ln = np.array([100_000, 77, 3, 99_999, 4_923, 0, 50_000], np.int64)
+    unit = np.array([3, 0, 3, 1, 0, 1, 4], np.int32)                # unit 2 has no segment
+    U = 5
+    base = _random_arena(rng, n, "bf16").to(cuda_device)
+    mon = Monitor(off, ln, dtype="bf16", segment_unit=unit, num_units=U, window=2, max_o=2,
+                  lock_len=1, device=0)
+    ctl = oracle.Controller(U, window=2, max_o=2, lock_len=1, alpha=(1.5, 1.1), beta=(1.5, 1.5))
+    stats = mon.new_stats()
+    try:
+        for t in range(4):
+            dev = (base.float() * float(1.0 + 0.37 * t)).to(torch.bfloat16)
+            norms = oracle.unit_norms_segmented(_host_view(dev), off, ln, unit, U)
+            assert norms[2] == 0.0
+            res = ctl.step(norms)
+            mask = mon.step(dev, stats=stats)
+            got = {k: v.cpu().numpy() for k, v in stats.items()}
+            got["mask"] = mask.cpu().numpy()
+            np.testing.assert_allclose(got["norm"], norms, rtol=RTOL, atol=0)
+            np.testing.assert_allclose(got["gnmr"], res.gnmr, rtol=RTOL, atol=0)
+    finally:
+        mon.close()
+        ctl.close()
+
+
 @pytest.mark.parametrize("seed", [1, 2])
 def test_tiny_more_seeds(seed, cuda_device):
     _run_lockstep(workloads.make("tiny", seed=seed, steps=120))

@@ -123,6 +123,27 @@ def test_norm_special_values():
     assert oracle.unit_norms(x * np.float32(8.0), [0], [777])[0] == 8.0 * base
 
 
+def test_segmented_norm_is_the_norm_of_the_concatenation():
+    """A block unit's norm (Sec. 3.4) is the L2 norm of all its segments'
+    elements together: compared with fsum over the concatenation."""
+    rng = np.random.default_rng(4)
+    x = (rng.standard_normal(20_000) * np.exp(2 * rng.standard_normal(20_000))).astype(np.float32)
+    off = np.array([0, 5000, 100, 7000, 19_000, 3, 12_000], np.int64)
+    ln = np.array([100, 2000, 900, 0, 1000, 4, 5000], np.int64)
+    unit = np.array([2, 0, 2, 1, 0, 2, 4], np.int32)          # unit 3 has no segment
+    for threads in (1, 3):
+        got = oracle.unit_norms_segmented(x, off, ln, unit, 5, threads)
+        for b in range(5):
+            seg = np.concatenate([x[o:o + n] for o, n, u in zip(off, ln, unit) if u == b] +
+                                 [np.zeros(0, np.float32)]).astype(np.float64)
+            assert got[b] == pytest.approx(math.sqrt(math.fsum(seg * seg)), rel=1e-12, abs=0.0)
+        assert got[3] == 0.0 and got[1] == 0.0
+    # one segment per unit: the plain per-unit norm
+    ident = np.arange(len(off), dtype=np.int32)
+    assert np.allclose(oracle.unit_norms_segmented(x, off, ln, ident, len(off)),
+                       oracle.unit_norms(x, off, ln), rtol=1e-15, atol=0)
+
+
 def test_norm_nonfinite_propagates():
     x = np.ones(10, np.float32)
     x[3] = np.inf

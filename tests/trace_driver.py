@@ -96,13 +96,17 @@ class LockstepTrace:
         torch = self.torch
         w = self.w
         torch.cuda.synchronize(self.dev)
-        if units is None:
+        if units is None or w.segment_unit is not None:
             if self._pinned is not None:
                 self._pinned.copy_(self.arena)
                 host = self._pinned
             else:
                 host = self.arena.cpu()
             view = host.view(torch.int16).numpy().view(np.uint16) if w.dtype == "bf16" else host.numpy()
+            if w.segment_unit is not None:
+                n = oracle.unit_norms_segmented(view, w.offsets, w.lengths, w.segment_unit,
+                                                w.num_units, self.threads)
+                return n if units is None else {u: n[u] for u in units}
             return oracle.unit_norms_threaded(view, w.offsets, w.lengths, self.threads)
         out = {}
         for u in units:
@@ -118,8 +122,9 @@ class LockstepTrace:
         which must write self.stats and return the mask) and returns
         (oracle norms, oracle result, GPU outputs as numpy)."""
         w = self.w
-        scales = w.scales[t].copy()
-        attempts = np.zeros(w.num_units, np.int32)
+        scales = w.scales[t].copy()                       # per segment (tensor)
+        attempts = np.zeros(w.num_segments, np.int32)
+        unit_attempts = np.zeros(w.num_units, np.int32)
         self.filler.fill(self.arena, t, scales, attempts)
         norms = self._host_norms()
         rec = StepRecord(t + 1, 0)
@@ -133,11 +138,17 @@ class LockstepTrace:
                 raise RuntimeError(f"step {t + 1}: no margin after {MAX_ATTEMPTS} redraws: {bad[:8]}")
             self.ctl.set_state(before)
             rec.attempts += 1
-            for u in bad:
-                attempts[u] += 1
-                scales[u] *= workloads.redraw_factor(w.seed, u, t, int(attempts[u]))
+            segs = []
+            for u in bad:                                  # one factor for all of a unit's tensors
+                unit_attempts[u] += 1
+                f = workloads.redraw_factor(w.seed, u, t, int(unit_attempts[u]))
+                mine = [u] if w.segment_unit is None else np.nonzero(w.segment_unit == u)[0].tolist()
+                for g in mine:
+                    attempts[g] += 1
+                    scales[g] *= f
+                segs.extend(mine)
             rec.repaired.extend(bad)
-            self.filler.fill(self.arena, t, scales, attempts, units=bad)
+            self.filler.fill(self.arena, t, scales, attempts, units=segs)
             for u, v in self._host_norms(bad).items():
                 norms[u] = v
         self.records.append(rec)

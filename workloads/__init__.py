@@ -42,8 +42,8 @@ IDS = {v: k for k, v in NAMES.items()}
 class Workload:
     name: str
     dtype: str                      # "f32" or "bf16"
-    offsets: np.ndarray             # int64 [U], elements
-    lengths: np.ndarray             # int64 [U]
+    offsets: np.ndarray             # int64 [S], elements, one per tensor (segment)
+    lengths: np.ndarray             # int64 [S]
     recoverable: np.ndarray         # uint8 [U]
     arena_elems: int
     steps: int
@@ -55,12 +55,20 @@ class Workload:
     warmup_steps: int
     eps: float
     seed: int
-    scales: np.ndarray              # float64 [steps, U]; 0 = unrouted (exact zeros)
+    scales: np.ndarray              # float64 [steps, S]; 0 = unrouted (exact zeros)
     kinds: list = field(default_factory=list)
+    segment_unit: np.ndarray | None = None   # int32 [S]: unit of each tensor; None = one each
+    group: str = "tensor"
+
+    @property
+    def num_segments(self) -> int:
+        return len(self.offsets)
 
     @property
     def num_units(self) -> int:
-        return len(self.offsets)
+        if self.segment_unit is None:
+            return len(self.offsets)
+        return int(self.segment_unit.max()) + 1
 
     @property
     def elem_bytes(self) -> int:
@@ -75,9 +83,12 @@ class Workload:
         return self.grad_elems * self.elem_bytes
 
     def monitor_kwargs(self) -> dict:
-        return dict(dtype=self.dtype, recoverable=self.recoverable, window=self.window,
-                    max_o=self.max_o, lock_len=self.lock_len, alpha=self.alpha, beta=self.beta,
-                    warmup_steps=self.warmup_steps, eps=self.eps)
+        kw = dict(dtype=self.dtype, recoverable=self.recoverable, window=self.window,
+                  max_o=self.max_o, lock_len=self.lock_len, alpha=self.alpha, beta=self.beta,
+                  warmup_steps=self.warmup_steps, eps=self.eps)
+        if self.segment_unit is not None:
+            kw.update(segment_unit=self.segment_unit, num_units=self.num_units)
+        return kw
 
     def controller_kwargs(self) -> dict:
         return dict(window=self.window, max_o=self.max_o, lock_len=self.lock_len,
@@ -128,10 +139,36 @@ def _linear_layout(layers, shapes, shrink):
     return np.array(lens, np.int64), kinds
 
 
-def make(config, seed: int = 0, shrink: int = 1, steps: int | None = None) -> Workload:
+def _grouping(cid, kinds, group):
+    """segment -> unit map for block-level units (Sec. 3.4): ``block`` makes
+    every transformer layer one unit; ``expert`` (MoE only) makes the attention
+    projections of a layer one unit and every expert's three matrices one."""
+    if group == "tensor":
+        return None
+    if cid not in (2, 3, 4):
+        raise ValueError("block/expert grouping applies to the model layouts (configs 2-4)")
+    keys = []
+    for k in kinds:
+        layer, name = k.split(".", 1)
+        if group == "block":
+            keys.append(layer)
+        elif group == "expert" and cid == 4:
+            keys.append(layer + "." + (name.split(".")[0] if "." in name else "attn"))
+        else:
+            raise ValueError(f"unknown grouping {group!r}")
+    ids, seen = [], {}
+    for key in keys:
+        ids.append(seen.setdefault(key, len(seen)))
+    return np.array(ids, np.int32)
+
+
+def make(config, seed: int = 0, shrink: int = 1, steps: int | None = None,
+         group: str = "tensor") -> Workload:
     """Builds workload ``config`` (1-5 or its name).  ``shrink`` divides every
     matrix dimension (configs 2-4) or unit length (configs 1, 5) to make a
-    small case with the same structure; ``steps`` overrides the step count."""
+    small case with the same structure; ``steps`` overrides the step count.
+    ``group`` = "tensor" (one unit per weight tensor), "block" (one unit per
+    transformer layer) or "expert" (MoE: attention and each expert grouped)."""
     cid = IDS.get(config, config)
     if cid not in NAMES:
         raise ValueError(f"unknown workload {config!r}")
@@ -210,11 +247,16 @@ def make(config, seed: int = 0, shrink: int = 1, steps: int | None = None) -> Wo
         warm = 0
     esize = 2 if dtype == "bf16" else 4
     offsets, arena_elems = _pack(lengths, esize)
-    return Workload(name=NAMES[cid], dtype=dtype, offsets=offsets, lengths=lengths,
-                    recoverable=np.ones(len(lengths), np.uint8), arena_elems=arena_elems,
-                    steps=T, window=window, max_o=max_o, lock_len=lock_len, alpha=alpha,
-                    beta=beta, warmup_steps=warm, eps=1e-8, seed=seed,
-                    scales=np.ascontiguousarray(scales), kinds=kinds)
+    seg_unit = _grouping(cid, kinds, group)
+    U = len(lengths) if seg_unit is None else int(seg_unit.max()) + 1
+    if seg_unit is not None:
+        max_o = max(1, min(max_o, U // 4))       # the budget scales with the coarser units
+    return Workload(name=NAMES[cid] + ("" if group == "tensor" else f"/{group}"), dtype=dtype,
+                    offsets=offsets, lengths=lengths, recoverable=np.ones(U, np.uint8),
+                    arena_elems=arena_elems, steps=T, window=window, max_o=max_o,
+                    lock_len=lock_len, alpha=alpha, beta=beta, warmup_steps=warm, eps=1e-8,
+                    seed=seed, scales=np.ascontiguousarray(scales), kinds=kinds,
+                    segment_unit=seg_unit, group=group)
 
 
 def redraw_factor(seed: int, unit: int, step: int, attempt: int) -> float:
@@ -260,7 +302,8 @@ def _load():
 
 class Filler:
     """Writes workload gradients into a device arena with the Philox fill
-    kernel.  One instance per (workload, device)."""
+    kernel, one weight tensor (segment) at a time.  One instance per
+    (workload, device)."""
 
     CHUNK = 1 << 20
 
@@ -270,9 +313,9 @@ class Filler:
         self.w = w
         self.device = torch.device(device)
         self._off = torch.from_numpy(w.offsets).to(self.device)
-        self._scale = torch.zeros(w.num_units, dtype=torch.float64, device=self.device)
-        self._attempt = torch.zeros(w.num_units, dtype=torch.int32, device=self.device)
-        self._all_tasks = self._tasks(np.arange(w.num_units))
+        self._scale = torch.zeros(w.num_segments, dtype=torch.float64, device=self.device)
+        self._attempt = torch.zeros(w.num_segments, dtype=torch.int32, device=self.device)
+        self._all_tasks = self._tasks(np.arange(w.num_segments))
 
     def _tasks(self, units):
         torch = self.torch
@@ -292,12 +335,13 @@ class Filler:
         return torch.full((self.w.arena_elems,), fill_value, dtype=dt, device=self.device)
 
     def fill(self, arena, step: int, scales=None, attempts=None, units=None, stream=None):
-        """Writes step ``step`` of every unit (or of ``units``) into arena.
-        ``scales``/``attempts`` default to the workload's scales and 0."""
+        """Writes step ``step`` of every segment (or of the segments listed in
+        ``units``) into arena.  ``scales``/``attempts`` (per segment) default
+        to the workload's scales and 0."""
         torch = self.torch
         sc = self.w.scales[step] if scales is None else scales
         self._scale.copy_(torch.from_numpy(np.ascontiguousarray(sc, np.float64)))
-        at = np.zeros(self.w.num_units, np.int32) if attempts is None else attempts
+        at = np.zeros(self.w.num_segments, np.int32) if attempts is None else attempts
         self._attempt.copy_(torch.from_numpy(np.ascontiguousarray(at, np.int32)))
         tu, ts, tc, n = self._all_tasks if units is None else self._tasks(units)
         st = stream.cuda_stream if stream is not None else torch.cuda.current_stream(self.device).cuda_stream
