@@ -41,6 +41,9 @@ def parse_args(argv=None):
     p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["gnmr", "reference"], default="gnmr")
+    p.add_argument("--kernel", choices=["step", "actuator"], default="step",
+                   help="step: the GNMR monitor (headline); actuator: the fake-quant actuator")
+    p.add_argument("--tokens", type=int, default=4096, help="tokens per microbatch (actuator)")
     p.add_argument("--workload", default="llama2-13b")
     p.add_argument("--group", default="tensor", choices=["tensor", "block", "expert"],
                    help="unit granularity: one per tensor, per transformer block, per MoE expert")
@@ -434,10 +437,91 @@ def run_gnmr(args):
         dist.destroy_process_group()
 
 
+def run_actuator(args):
+    """Fake-quant actuator over the saved input activations of every linear of
+    the LLaMA-2-13B layout for one microbatch: unit b is a [tokens, in_features]
+    bf16 block; 10 % of units take the recovery format (E4M3), the rest the
+    low-cost one (E2M1).  Algorithmic bytes: one read and one write."""
+    import torch
+    import workloads
+    from paper_2606_00539_gb300 import _native as N
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = workloads.make("llama2-13b", shrink=args.shrink)
+    in_features = np.array([int(k) for k in _in_features(w)], np.int64)
+    rows = np.full(w.num_units, args.tokens, np.int64)
+    cols = in_features
+    off = np.concatenate([[0], np.cumsum(rows * cols)[:-1]]).astype(np.int64)
+    total = int((rows * cols).sum())
+    acts = torch.empty(total, dtype=torch.bfloat16, device=dev)
+    gen = torch.Generator(device=dev).manual_seed(0)
+    for s0 in range(0, total, 1 << 28):
+        n = min(1 << 28, total - s0)
+        acts[s0:s0 + n] = torch.randn(n, generator=gen, device=dev).to(torch.bfloat16)
+    out = torch.empty_like(acts)
+    mask = (torch.rand(w.num_units, generator=gen, device=dev) < 0.1).to(torch.uint8)
+    h = N.gnmr_actuator_create(off, rows, cols, N.GNMR_DTYPE_BF16, 0)
+    stream = torch.cuda.Stream(dev)
+    sp = stream.cuda_stream
+    for _ in range(args.warmup):
+        N.gnmr_actuator_apply(h, acts.data_ptr(), out.data_ptr(), total, mask.data_ptr(),
+                              N.GNMR_FQ_E2M1, N.GNMR_FQ_E4M3, sp)
+    stream.synchronize()
+    sampler = ClockSampler(0)
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    torch.cuda.synchronize(dev)
+    wall0 = time.time()
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        N.gnmr_actuator_apply(h, acts.data_ptr(), out.data_ptr(), total, mask.data_ptr(),
+                              N.GNMR_FQ_E2M1, N.GNMR_FQ_E4M3, sp)
+        ev[i][1].record(stream)
+    stream.synchronize()
+    wall1 = time.time()
+    sampler.stop()
+    N.gnmr_actuator_destroy(h)
+    per_ms = [a.elapsed_time(b) for a, b in ev]
+    ms = statistics.mean(per_ms)
+    nbytes = 2 * total * 2
+    peak, peak_kind = measured_peaks()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    print(json.dumps({
+        "metric": "GNMR recovery actuator: per-token fake quantization GB/s (read + write)",
+        "value": round(gbs, 2), "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"llama2-13b input activations, {w.num_units} units x "
+                               f"{args.tokens} tokens ({total} bf16 elements)",
+                   "formats": "E2M1 low-cost, E4M3 recovery (10 % of units)",
+                   "l2": "inputs larger than L2 (no flush)"},
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(gbs / peak, 4), "traffic": None,
+                     "algorithmic_bytes": nbytes, "peak_source": f"{peak_kind} hbm_gbs",
+                     "kernel": "fake_quant_kernel<bf16>", "kernel_ms_min": round(min(per_ms), 4)},
+        "gpu_launches": args.steps, "clocks": sampler.summary(wall0, wall1),
+    }), flush=True)
+
+
+def _in_features(w):
+    """Input width of every linear of a LLaMA layout (the saved activation of
+    x @ W^T is [tokens, in_features])."""
+    d = {"llama2-13b": (5120, 13824), "llama2-1.3b": (2048, 5504)}[w.name.split("/")[0]]
+    out = []
+    for k in w.kinds:
+        name = k.split(".", 1)[1]
+        out.append(d[1] if name == "down" else d[0])
+    return out
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.impl == "reference":
         run_reference(args)
+    elif args.kernel == "actuator":
+        run_actuator(args)
     else:
         run_gnmr(args)
 

@@ -207,8 +207,9 @@ gnmr_status gnmr_destroy(gnmr_handle *h);
 /* Static text for a status code. */
 const char *gnmr_status_string(gnmr_status s);
 
-/* Detail of the last failure on h; with h == NULL, of the last failed
- * gnmr_create or gnmr_unit_norms_static on the calling thread.  Valid until the next call on h (or
+/* Detail of the last failure on h; with h == NULL, of the last failed call
+ * without a handle (gnmr_create, the actuator calls, gnmr_unit_norms_static)
+ * on the calling thread.  Valid until the next call on h (or
  * create on this thread); never NULL. */
 const char *gnmr_last_error(const gnmr_handle *h);
 
@@ -225,6 +226,46 @@ const char *gnmr_last_error(const gnmr_handle *h);
 gnmr_status gnmr_plan_partition(int32_t num_units, const int64_t *lengths, int32_t dtype,
                                 int32_t max_warps, int32_t *num_warps, int32_t *run_unit,
                                 int64_t *run_pos, int32_t *first_warp, int32_t *num_parts);
+
+/* ---- Recovery actuator (App. E.2; the stress bench of Sec. 5.1) --------
+ * The mask decides, per unit, which path the unit's saved activations take:
+ * the low-cost format or the higher-fidelity recovery format.  The actuator
+ * fake-quantizes each unit's activations token by token: for every row,
+ * amax = max |x|, inv = fmax / amax, scale = amax / fmax, and
+ * y = round(x * inv) * scale, where round() gives the nearest value
+ * representable in the format (ties to the even code, saturating at fmax).
+ * All of this is fp32 arithmetic.  Rows whose amax is 0 or that hold a NaN or
+ * Inf are copied unchanged. */
+typedef enum gnmr_fq_format {
+    GNMR_FQ_NONE = 0,   /* copy (no quantization) */
+    GNMR_FQ_E2M1 = 1,   /* 4-bit: 2 exponent bits (bias 1), 1 mantissa bit, max 6 */
+    GNMR_FQ_E3M2 = 2,   /* 6-bit: bias 3, max 28 */
+    GNMR_FQ_E4M3 = 3,   /* 8-bit: bias 7, max 448 */
+    GNMR_FQ_E5M2 = 4    /* 8-bit: bias 15, max 57344 */
+} gnmr_fq_format;
+
+typedef struct gnmr_actuator gnmr_actuator;
+
+/* Activation layout: unit b's activations are a row-major [rows[b] x
+ * cols[b]] block (one row per token) starting at element offsets[b] of a flat
+ * buffer of `dtype` (host arrays, copied).  Errors: GNMR_ERR_INVALID_ARG,
+ * GNMR_ERR_CUDA, GNMR_ERR_OOM; detail via gnmr_last_error(NULL). */
+gnmr_status gnmr_actuator_create(int32_t num_units, const int64_t *offsets, const int64_t *rows,
+                                 const int64_t *cols, int32_t dtype, int32_t device,
+                                 gnmr_actuator **out);
+
+/* Fake-quantizes every unit's activations from d_in into d_out (device, same
+ * layout; d_out == d_in works in place) on `stream`: unit b uses
+ * recovery_format if d_mask[b] != 0, else lowcost_format (d_mask: device
+ * uint8 [num_units] as written by gnmr_step, or NULL = low-cost for all).
+ * arena_elems bounds both buffers.  Errors: GNMR_ERR_INVALID_ARG,
+ * GNMR_ERR_LAYOUT, GNMR_ERR_CUDA. */
+gnmr_status gnmr_actuator_apply(gnmr_actuator *a, const void *d_in, void *d_out, int64_t arena_elems,
+                                const uint8_t *d_mask, int32_t lowcost_format,
+                                int32_t recovery_format, void *stream);
+
+/* Frees the actuator (waits for its device).  NULL is accepted. */
+gnmr_status gnmr_actuator_destroy(gnmr_actuator *a);
 
 /* Allocation-free per-unit norms.  The paper has no counterpart: this is a
  * deployment variant of the first stage of gnmr_step.

@@ -41,8 +41,8 @@ def build(force: bool = False) -> str:
              or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC))
     if force or stale:
         tmp = _LIB_PATH + f".tmp{os.getpid()}"
-        subprocess.check_call(["gcc", "-O2", "-std=c11", "-Wall", "-shared", "-fPIC",
-                               "-o", tmp, _SRC, "-lm"])
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-Wall", "-shared",
+                               "-fPIC", "-o", tmp, _SRC, "-lm"])
         os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
 
@@ -58,6 +58,10 @@ def _load():
     lib.oracle_unit_norms_segmented.argtypes = [P, ctypes.c_int, P, P, P, ctypes.c_int64,
                                                 ctypes.c_int32, P]
     lib.oracle_unit_norms_segmented.restype = ctypes.c_int
+    lib.oracle_fq_round.argtypes = [ctypes.c_float, ctypes.c_int]
+    lib.oracle_fq_round.restype = ctypes.c_float
+    lib.oracle_fake_quant.argtypes = [P, P, ctypes.c_int, ctypes.c_int64, ctypes.c_int64, ctypes.c_int]
+    lib.oracle_fake_quant.restype = ctypes.c_int
     lib.oracle_ctl_create.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                       ctypes.c_int32, ctypes.c_int64, ctypes.c_double,
                                       ctypes.c_double, ctypes.c_double, ctypes.c_double,
@@ -171,6 +175,28 @@ def unit_norms_segmented(arena: np.ndarray, offsets, lengths, segment_unit, num_
     else:
         with ThreadPoolExecutor(max_workers=threads) as ex:
             list(ex.map(run, range(threads)))
+    return out
+
+
+FQ_NONE, FQ_E2M1, FQ_E3M2, FQ_E4M3, FQ_E5M2 = 0, 1, 2, 3, 4
+
+
+def fq_round(v: float, code: int) -> float:
+    """Nearest value of minifloat format ``code`` to the fp32 value v."""
+    return float(_load().oracle_fq_round(float(v), int(code)))
+
+
+def fake_quant(x: np.ndarray, code: int) -> np.ndarray:
+    """Per-token fake quantization (App. E.2) of a [rows, cols] float32 array
+    or uint16 array of bfloat16 bits; returns a new array of the same kind."""
+    x = np.ascontiguousarray(x)
+    if x.ndim != 2:
+        raise ValueError("x must be [rows, cols]")
+    out = np.empty_like(x)
+    rc = _load().oracle_fake_quant(_ptr(x), _ptr(out), _arena_dtype(x), x.shape[0], x.shape[1],
+                                   int(code))
+    if rc != 0:
+        raise ValueError("bad format or dtype")
     return out
 
 

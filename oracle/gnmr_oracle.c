@@ -25,9 +25,19 @@
  *   - alpha_t, beta_t: the *_init values for t <= warmup_steps, the *_main
  *     values after, unless the caller overrides them for the step.
  *
- * Build: gcc -O2 -shared -fPIC -o liboracle_gnmr.so gnmr_oracle.c -lm
- * (no fast-math: every sum below runs in the order written).
+ *   - The recovery actuator's fake quantization (App. E.2, the low-cost
+ *     activation path of the stress bench in Sec. 5.1): per token row, scale
+ *     into the format's range, round to the nearest representable value,
+ *     rescale.  The paper fixes no precision for this arithmetic; the reading
+ *     taken is fp32 throughout (inv = fmax / amax, v = x * inv, y = q * (amax /
+ *     fmax)), ties to the even code, saturation at fmax, rows whose max is 0
+ *     or that hold a NaN or Inf left unchanged.
+ *
+ * Build: gcc -O2 -std=c11 -ffp-contract=off -shared -fPIC -o liboracle_gnmr.so
+ * gnmr_oracle.c -lm (no fast-math, no fused multiply-add: every operation
+ * below rounds as written).
  */
+#include <float.h>
 #include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
@@ -335,4 +345,108 @@ void oracle_ctl_set_state(oracle_ctl *c, const double *A, const int64_t *k,
     memcpy(c->qlen, qlen, u * sizeof(int32_t));
     memcpy(c->lock, lock, u * sizeof(int32_t));
     c->t = t;
+}
+
+/* ---- recovery actuator: fake quantization (App. E.2) ------------------- */
+
+/* Minifloat formats: exponent bits, mantissa bits, exponent bias, largest
+ * finite value.  1 = E2M1 (FP4), 2 = E3M2 (FP6), 3 = E4M3, 4 = E5M2 (FP8). */
+typedef struct {
+    int mbits;
+    int emin;      /* exponent of the smallest normal value, 1 - bias */
+    float fmax;
+} fq_format;
+
+static int fq_lookup(int code, fq_format *f)
+{
+    switch (code) {
+    case 1: f->mbits = 1; f->emin = 1 - 1; f->fmax = 6.0f; return 0;
+    case 2: f->mbits = 2; f->emin = 1 - 3; f->fmax = 28.0f; return 0;
+    case 3: f->mbits = 3; f->emin = 1 - 7; f->fmax = 448.0f; return 0;
+    case 4: f->mbits = 2; f->emin = 1 - 15; f->fmax = 57344.0f; return 0;
+    default: return 1;
+    }
+}
+
+/* Nearest representable value of the format to v (ties to the even code),
+ * saturating at +-fmax.  Values with exponent e >= emin are spaced
+ * 2^(e - mbits); below 2^emin (subnormals) the spacing stays 2^(emin - mbits). */
+float oracle_fq_round(float v, int code)
+{
+    fq_format f;
+    if (fq_lookup(code, &f))
+        return v;
+    float a = fabsf(v);
+    float r;
+    if (a >= f.fmax) {
+        r = f.fmax;
+    } else if (a == 0.0f) {
+        r = 0.0f;
+    } else {
+        int e2;
+        frexpf(a, &e2);               /* a = m * 2^e2, m in [0.5, 1) */
+        int e = e2 - 1;               /* floor(log2 a) */
+        if (e < f.emin)
+            e = f.emin;
+        float quantum = ldexpf(1.0f, e - f.mbits);
+        r = rintf(a / quantum) * quantum;
+    }
+    return copysignf(r, v);
+}
+
+static float bf16_to_float_row(const uint16_t *p, int64_t i)
+{
+    uint32_t bits = ((uint32_t)p[i]) << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return f;
+}
+
+/* float -> bfloat16, round to nearest even (NaN kept as a quiet NaN). */
+static uint16_t float_to_bf16_bits(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7fffffffu) > 0x7f800000u)
+        return (uint16_t)((u >> 16) | 0x40u);
+    u += 0x7fffu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+/* Fake-quantizes a row-major [rows x cols] tensor, token (row) by token:
+ * amax = max |x|; inv = fmax / amax; scale = amax / fmax; y = round(x * inv)
+ * * scale.  code 0 copies.  in and out may be the same buffer. */
+int oracle_fake_quant(const void *in, void *out, int dtype, int64_t rows, int64_t cols, int code)
+{
+    fq_format f = {0, 0, 1.0f};
+    if (code != 0 && fq_lookup(code, &f))
+        return 1;
+    if (dtype != ORACLE_DTYPE_F32 && dtype != ORACLE_DTYPE_BF16)
+        return 1;
+    for (int64_t r = 0; r < rows; ++r) {
+        float amax = 0.0f;
+        int nonfinite = 0;
+        for (int64_t c = 0; c < cols; ++c) {
+            float x = dtype == ORACLE_DTYPE_F32 ? ((const float *)in)[r * cols + c]
+                                               : bf16_to_float_row((const uint16_t *)in, r * cols + c);
+            if (!isfinite(x))
+                nonfinite = 1;
+            else if (fabsf(x) > amax)
+                amax = fabsf(x);
+        }
+        int keep = code == 0 || amax == 0.0f || nonfinite;
+        float inv = keep ? 1.0f : f.fmax / amax;
+        float scale = keep ? 1.0f : amax / f.fmax;
+        for (int64_t c = 0; c < cols; ++c) {
+            int64_t i = r * cols + c;
+            float x = dtype == ORACLE_DTYPE_F32 ? ((const float *)in)[i]
+                                               : bf16_to_float_row((const uint16_t *)in, i);
+            float y = keep ? x : oracle_fq_round(x * inv, code) * scale;
+            if (dtype == ORACLE_DTYPE_F32)
+                ((float *)out)[i] = y;
+            else
+                ((uint16_t *)out)[i] = keep ? ((const uint16_t *)in)[i] : float_to_bf16_bits(y);
+        }
+    }
+    return 0;
 }

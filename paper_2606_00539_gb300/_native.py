@@ -21,6 +21,8 @@ GNMR_ERR_STATE = 5
 GNMR_DTYPE_F32 = 0
 GNMR_DTYPE_BF16 = 1
 
+GNMR_FQ_NONE, GNMR_FQ_E2M1, GNMR_FQ_E3M2, GNMR_FQ_E4M3, GNMR_FQ_E5M2 = 0, 1, 2, 3, 4
+
 _P = ctypes.c_void_p
 
 
@@ -93,6 +95,11 @@ PROTOTYPES = {
                                            _P, _P, _P, _P, _P]),
     "gnmr_unit_norms_static": (ctypes.c_int, [_P, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                               _P, _P, _P, _P]),
+    "gnmr_actuator_create": (ctypes.c_int, [ctypes.c_int32, _P, _P, _P, ctypes.c_int32, ctypes.c_int32,
+                                            ctypes.POINTER(_P)]),
+    "gnmr_actuator_apply": (ctypes.c_int, [_P, _P, _P, ctypes.c_int64, _P, ctypes.c_int32, ctypes.c_int32,
+                                           _P]),
+    "gnmr_actuator_destroy": (ctypes.c_int, [_P]),
     "gnmr_step_partials": (ctypes.c_int, [_P, _P, ctypes.c_int64, _P, _P]),
     "gnmr_finish": (ctypes.c_int, [_P, _P, _P, _P, ctypes.POINTER(gnmr_stats)]),
     "gnmr_get_state": (ctypes.c_int, [_P, _P, _P, ctypes.c_int64, ctypes.POINTER(ctypes.c_int64)]),
@@ -211,3 +218,26 @@ def gnmr_plan_partition(lengths, dtype: int, max_warps: int):
     _check(st, None)
     n = nw.value
     return run_unit[:n + 1], run_pos[:n + 1], first, parts
+
+
+def gnmr_actuator_create(offsets, rows, cols, dtype: int, device: int = 0) -> int:
+    import numpy as np
+    off = np.ascontiguousarray(offsets, dtype=np.int64)
+    r = np.ascontiguousarray(rows, dtype=np.int64)
+    c = np.ascontiguousarray(cols, dtype=np.int64)
+    h = _P()
+    st = load().gnmr_actuator_create(len(off), off.ctypes.data, r.ctypes.data, c.ctypes.data,
+                                     int(dtype), int(device), ctypes.byref(h))
+    _check(st, None)
+    return h.value
+
+
+def gnmr_actuator_apply(handle: int, d_in: int, d_out: int, arena_elems: int, d_mask,
+                        lowcost_format: int, recovery_format: int, stream: int = 0) -> None:
+    st = load().gnmr_actuator_apply(handle, d_in, d_out, int(arena_elems), d_mask,
+                                    int(lowcost_format), int(recovery_format), stream)
+    _check(st, None)
+
+
+def gnmr_actuator_destroy(handle: int) -> None:
+    _check(load().gnmr_actuator_destroy(handle), None)

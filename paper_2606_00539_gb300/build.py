@@ -18,7 +18,7 @@ BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(PKG, "libgnmr.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-CUDA_SOURCES = ["gnmr_kernels.cu", "gnmr_static.cu"]
+CUDA_SOURCES = ["gnmr_kernels.cu", "gnmr_static.cu", "gnmr_actuator.cu"]
 CXX_SOURCES = ["gnmr_api.cpp", "gnmr_plan.cpp"]
 HEADERS = ["gnmr_internal.h"]
 
