@@ -72,6 +72,13 @@ def _load():
     lib.oracle_ctl_step.argtypes = [P, P, ctypes.c_double, ctypes.c_double,
                                     P, P, P, P, P, P]
     lib.oracle_ctl_step.restype = ctypes.c_int
+    lib.oracle_ctl_set_policy.argtypes = [P, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64,
+                                          ctypes.c_double]
+    lib.oracle_ctl_set_policy.restype = ctypes.c_int
+    lib.oracle_ctl_get_policy_state.argtypes = [P, P, P]
+    lib.oracle_ctl_get_policy_state.restype = None
+    lib.oracle_delta_mem.argtypes = [P, P, ctypes.c_int32]
+    lib.oracle_delta_mem.restype = ctypes.c_double
     lib.oracle_ctl_get_state.argtypes = [P, P, P, P, P, P, P]
     lib.oracle_ctl_get_state.restype = None
     lib.oracle_ctl_set_state.argtypes = [P, P, P, P, P, P, ctypes.c_int64]
@@ -178,7 +185,17 @@ def unit_norms_segmented(arena: np.ndarray, offsets, lengths, segment_unit, num_
     return out
 
 
+POLICY_ACTIVE_CAP, POLICY_ADMISSION_CAP, POLICY_STATIC_TOP = 0, 1, 2
+
 FQ_NONE, FQ_E2M1, FQ_E3M2, FQ_E4M3, FQ_E5M2 = 0, 1, 2, 3, 4
+
+
+def delta_mem(mask, cost) -> float:
+    """Eq. generic-memory-bound: the extra saved-activation memory of the
+    units on the recovery path, Delta M_t = sum over b in A_t of c_b."""
+    m = np.ascontiguousarray(mask, dtype=np.uint8)
+    c = np.ascontiguousarray(cost, dtype=np.float64)
+    return float(_load().oracle_delta_mem(_ptr(m), _ptr(c), len(m)))
 
 
 def fq_round(v: float, code: int) -> float:
@@ -218,7 +235,9 @@ class Controller:
 
     def __init__(self, num_units: int, window: int, max_o: int, lock_len: int,
                  alpha=(1.5, 1.5), beta=(1.5, 1.5), warmup_steps: int = 0,
-                 eps: float = 1e-8, recoverable=None):
+                 eps: float = 1e-8, recoverable=None, policy: int = 0,
+                 forced_recovery_steps: int = 0, static_warmup_steps: int = 0,
+                 static_fraction: float = 0.25):
         self.num_units = int(num_units)
         self.window = int(window)
         lib = _load()
@@ -233,6 +252,9 @@ class Controller:
                                         None if rec is None else _ptr(rec))
         if not self._h:
             raise ValueError("invalid oracle controller configuration")
+        if lib.oracle_ctl_set_policy(self._h, int(policy), int(forced_recovery_steps),
+                                     int(static_warmup_steps), float(static_fraction)) != 0:
+            raise ValueError("invalid oracle policy")
 
     def close(self):
         if getattr(self, "_h", None):
@@ -266,6 +288,12 @@ class Controller:
         st["Q"] = st["Q"].reshape(U, w)
         st["t"] = int(t.value)
         return st
+
+    def policy_state(self) -> dict:
+        active = np.empty(self.num_units, np.uint8)
+        gsum = np.empty(self.num_units, np.float64)
+        _load().oracle_ctl_get_policy_state(self._h, _ptr(active), _ptr(gsum))
+        return dict(active=active, gsum=gsum)
 
     def set_state(self, st: dict) -> None:
         A = np.ascontiguousarray(st["A"], np.float64)

@@ -137,7 +137,18 @@ typedef struct {
     int32_t *qlen;
     int32_t *lock;
     int32_t *cand;       /* scratch for Algorithm 2 */
+    /* policy variants (see oracle_ctl_set_policy) */
+    int32_t policy;
+    int64_t forced_steps;
+    int64_t static_warmup;
+    double static_fraction;
+    uint8_t *active;     /* A_{t-1}: on the recovery path at the previous step */
+    double *gsum;        /* sum of GNMR over the static policy's warm-up */
 } oracle_ctl;
+
+#define ORACLE_POLICY_ACTIVE_CAP 0
+#define ORACLE_POLICY_ADMISSION_CAP 1
+#define ORACLE_POLICY_STATIC_TOP 2
 
 void oracle_ctl_destroy(oracle_ctl *c)
 {
@@ -150,6 +161,8 @@ void oracle_ctl_destroy(oracle_ctl *c)
     free(c->qlen);
     free(c->lock);
     free(c->cand);
+    free(c->active);
+    free(c->gsum);
     free(c);
 }
 
@@ -182,13 +195,43 @@ oracle_ctl *oracle_ctl_create(int32_t num_units, int32_t window, int32_t max_o,
     c->qlen = (int32_t *)calloc(u, sizeof(int32_t));
     c->lock = (int32_t *)calloc(u, sizeof(int32_t));
     c->cand = (int32_t *)calloc(u, sizeof(int32_t));
-    if (!c->recoverable || !c->A || !c->k || !c->Q || !c->qlen || !c->lock || !c->cand) {
+    c->active = (uint8_t *)calloc(u, 1);
+    c->gsum = (double *)calloc(u, sizeof(double));
+    c->static_fraction = 0.25;
+    if (!c->recoverable || !c->A || !c->k || !c->Q || !c->qlen || !c->lock || !c->cand ||
+        !c->active || !c->gsum) {
         oracle_ctl_destroy(c);
         return NULL;
     }
     for (size_t b = 0; b < u; ++b)
         c->recoverable[b] = recoverable ? (recoverable[b] != 0) : 1;
     return c;
+}
+
+/* Policy variants (readings of passages the paper states loosely):
+ *   ORACLE_POLICY_ACTIVE_CAP (0, Algorithm 2): |A_t| <= maxO.
+ *   ORACLE_POLICY_ADMISSION_CAP (1, the Remark on the maxO budget): only newly
+ *     admitted units are capped.  Candidates that were active at t-1 stay
+ *     active; of the other candidates the maxO with the largest R (ties by
+ *     index) are admitted.  |A_t| may exceed maxO.
+ *   ORACLE_POLICY_STATIC_TOP (2, the ADAPT-style baseline of App. E.4): for
+ *     t <= static_warmup every recoverable unit is on the recovery path and
+ *     GNMR is summed per unit; at t = static_warmup + 1 the
+ *     ceil(static_fraction * |B_rec|) recoverable units with the largest sum
+ *     (ties by index) are fixed on the recovery path for good.
+ * forced_steps (App. E.7): for t <= forced_steps every recoverable unit is on
+ * the recovery path (statistics still update, locks stay as they are). */
+int oracle_ctl_set_policy(oracle_ctl *c, int32_t policy, int64_t forced_steps,
+                          int64_t static_warmup, double static_fraction)
+{
+    if (policy < 0 || policy > 2 || forced_steps < 0 || static_warmup < 0 ||
+        !(static_fraction >= 0.0 && static_fraction <= 1.0))
+        return 1;
+    c->policy = policy;
+    c->forced_steps = forced_steps;
+    c->static_warmup = static_warmup;
+    c->static_fraction = static_fraction;
+    return 0;
 }
 
 /* Algorithm 1 for one unit: returns GNMR and Delta-GNMR through g and d, and
@@ -285,21 +328,94 @@ int oracle_ctl_step(oracle_ctl *c, const double *norms, double alpha_override,
         risk[b] = (x > y) ? x : y;
     }
 
+    int32_t nrec = 0;
+    for (int32_t b = 0; b < U; ++b)
+        nrec += c->recoverable[b];
+
+    if (c->policy == ORACLE_POLICY_STATIC_TOP && c->t <= c->static_warmup)
+        for (int32_t b = 0; b < U; ++b)
+            if (c->recoverable[b])
+                c->gsum[b] += gnmr[b];
+
+    /* Every recoverable unit on the recovery path: forced warm-up, or the
+     * static policy's warm-up. */
+    if (c->t <= c->forced_steps ||
+        (c->policy == ORACLE_POLICY_STATIC_TOP && c->t <= c->static_warmup)) {
+        for (int32_t b = 0; b < U; ++b) {
+            mask[b] = c->recoverable[b];
+            c->active[b] = c->recoverable[b];
+            lock_out[b] = c->lock[b];
+        }
+        counts[0] = 0;
+        counts[1] = nrec;
+        return 0;
+    }
+
+    /* Static policy: choose once, then keep. */
+    if (c->policy == ORACLE_POLICY_STATIC_TOP) {
+        int32_t pool = 0;
+        if (c->t == c->static_warmup + 1) {
+            for (int32_t b = 0; b < U; ++b)
+                if (c->recoverable[b])
+                    c->cand[pool++] = b;
+            g_sort_r = c->gsum;
+            qsort(c->cand, (size_t)pool, sizeof(int32_t), by_risk_then_index);
+            int32_t keep = (int32_t)ceil(c->static_fraction * (double)nrec);
+            if (keep > pool)
+                keep = pool;
+            for (int32_t b = 0; b < U; ++b)
+                c->active[b] = 0;
+            for (int32_t i = 0; i < keep; ++i)
+                c->active[c->cand[i]] = 1;
+        }
+        int32_t nfixed = 0;
+        for (int32_t b = 0; b < U; ++b) {
+            mask[b] = c->active[b];
+            nfixed += c->active[b];
+            lock_out[b] = c->lock[b];
+        }
+        counts[0] = pool;
+        counts[1] = nfixed;
+        return 0;
+    }
+
     /* C_t = {b : R > 1} U {b : Lock_b > 0}, over recoverable units only. */
     int32_t ncand = 0;
     for (int32_t b = 0; b < U; ++b)
         if (c->recoverable[b] && (risk[b] > 1.0 || c->lock[b] > 0))
             c->cand[ncand++] = b;
 
-    /* A_t = Top_maxO(C_t; R): sort by R descending, index ascending. */
-    g_sort_r = risk;
-    qsort(c->cand, (size_t)ncand, sizeof(int32_t), by_risk_then_index);
-    int32_t nsel = ncand < c->max_o ? ncand : c->max_o;
-
     for (int32_t b = 0; b < U; ++b)
         mask[b] = 0;
-    for (int32_t i = 0; i < nsel; ++i)
-        mask[c->cand[i]] = 1;
+    int32_t nsel = 0;
+    if (c->policy == ORACLE_POLICY_ADMISSION_CAP) {
+        /* candidates active at t-1 stay; at most maxO new ones are admitted */
+        int32_t nnew = 0;
+        for (int32_t i = 0; i < ncand; ++i) {
+            int32_t b = c->cand[i];
+            if (c->active[b]) {
+                mask[b] = 1;
+                ++nsel;
+            } else {
+                c->cand[nnew++] = b;
+            }
+        }
+        g_sort_r = risk;
+        qsort(c->cand, (size_t)nnew, sizeof(int32_t), by_risk_then_index);
+        int32_t admit = nnew < c->max_o ? nnew : c->max_o;
+        for (int32_t i = 0; i < admit; ++i)
+            mask[c->cand[i]] = 1;
+        nsel += admit;
+    } else {
+        /* A_t = Top_maxO(C_t; R): sort by R descending, index ascending. */
+        g_sort_r = risk;
+        qsort(c->cand, (size_t)ncand, sizeof(int32_t), by_risk_then_index);
+        nsel = ncand < c->max_o ? ncand : c->max_o;
+        for (int32_t i = 0; i < nsel; ++i)
+            mask[c->cand[i]] = 1;
+    }
+    for (int32_t b = 0; b < U; ++b)
+        c->active[b] = mask[b];
 
     /* Lock bookkeeping of Algorithm 2. */
     for (int32_t b = 0; b < U; ++b) {
@@ -449,4 +565,22 @@ int oracle_fake_quant(const void *in, void *out, int dtype, int64_t rows, int64_
         }
     }
     return 0;
+}
+
+/* Policy state for checkpoint tests: active[U] (A_{t-1}) and gsum[U]. */
+void oracle_ctl_get_policy_state(const oracle_ctl *c, uint8_t *active, double *gsum)
+{
+    memcpy(active, c->active, (size_t)c->num_units);
+    memcpy(gsum, c->gsum, (size_t)c->num_units * sizeof(double));
+}
+
+/* Eq. generic-memory-bound: Delta M_t = sum over b in A_t of c_b, summed in
+ * unit order. */
+double oracle_delta_mem(const uint8_t *mask, const double *cost, int32_t num_units)
+{
+    double s = 0.0;
+    for (int32_t b = 0; b < num_units; ++b)
+        if (mask[b])
+            s += cost[b];
+    return s;
 }

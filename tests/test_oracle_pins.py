@@ -20,13 +20,20 @@ def _f(x):
     return float(x)
 
 
+def policy_kwargs(cfg):
+    return dict(policy=int(cfg.get("policy", 0)), forced_recovery_steps=int(cfg.get("forced", 0)),
+                static_warmup_steps=int(cfg.get("static_warmup", 0)),
+                static_fraction=_f(cfg.get("static_fraction", Fraction(1, 4))))
+
+
 def _controller_from(cfg):
     return oracle.Controller(
         int(cfg["units"]), int(cfg["window"]), int(cfg["max_o"]), int(cfg["lock_len"]),
         alpha=(_f(cfg["alpha_init"]), _f(cfg["alpha_main"])),
         beta=(_f(cfg["beta_init"]), _f(cfg["beta_main"])),
         warmup_steps=int(cfg["warmup"]), eps=_f(cfg["eps"]),
-        recoverable=np.array([int(x) for x in cfg["recoverable"]], np.uint8))
+        recoverable=np.array([int(x) for x in cfg["recoverable"]], np.uint8),
+        **policy_kwargs(cfg))
 
 
 def _close(got, want, rel=1e-12):
@@ -73,9 +80,11 @@ def test_hand_trace_fixtures_are_consistent():
                 r = max(g / a if not isinstance(g, float) else g,
                         d / b_ if not isinstance(d, float) else d)
                 assert r == st.risk[b], (tr.name, st.t, b)
-            cand = [b for b in range(int(cfg["units"]))
-                    if cfg["recoverable"][b] and (st.risk[b] > 1 or prev_lock[b] > 0)]
-            assert cand == st.candidates, (tr.name, st.t)
+            pool_formed = st.t > cfg.get("forced", 0) and cfg.get("policy", 0) != 2
+            if pool_formed:
+                cand = [b for b in range(int(cfg["units"]))
+                        if cfg["recoverable"][b] and (st.risk[b] > 1 or prev_lock[b] > 0)]
+                assert cand == st.candidates, (tr.name, st.t)
             prev_lock = st.lock_after
 
 
@@ -142,6 +151,20 @@ def test_segmented_norm_is_the_norm_of_the_concatenation():
     ident = np.arange(len(off), dtype=np.int32)
     assert np.allclose(oracle.unit_norms_segmented(x, off, ln, ident, len(off)),
                        oracle.unit_norms(x, off, ln), rtol=1e-15, atol=0)
+
+
+def test_delta_mem_is_the_cost_of_the_active_set():
+    """Eq. generic-memory-bound: Delta M_t = sum of c_b over b in A_t, at most
+    maxO * c_max under the active cap."""
+    rng = np.random.default_rng(12)
+    U = 40
+    cost = rng.uniform(1, 100, U)
+    ctl = oracle.Controller(U, 3, 5, 2, alpha=(1.05, 1.05), beta=(1.05, 1.05))
+    for norms in _spiky_trace(rng, 30, U, spike_p=0.3):
+        res = ctl.step(norms)
+        dm = oracle.delta_mem(res.mask, cost)
+        assert dm == pytest.approx(math.fsum(cost[b] for b in range(U) if res.mask[b]), rel=1e-15)
+        assert dm <= 5 * cost.max()
 
 
 def test_norm_nonfinite_propagates():
@@ -354,3 +377,63 @@ def test_gnmr_exceedance_decreases_on_iid_norms():
         res = ctl.step(rng.exponential(1.0, U) + 1.0)
         hits[t] = np.mean(res.gnmr >= 1.6)
     assert hits[1:5].mean() > hits[40:].mean()
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_admission_cap_invariants(seed):
+    """Remark on the maxO budget: only newly admitted units are capped."""
+    rng = np.random.default_rng(300 + seed)
+    U, max_o = 30, 3
+    rec = (rng.random(U) < 0.8).astype(np.uint8)
+    ctl = oracle.Controller(U, 3, max_o, 2, alpha=(1.1, 1.1), beta=(1.1, 1.1), recoverable=rec,
+                            policy=oracle.POLICY_ADMISSION_CAP)
+    prev_active = np.zeros(U, bool)
+    lock_prev = np.zeros(U, np.int32)
+    for norms in _spiky_trace(rng, 40, U, spike_p=0.2):
+        res = ctl.step(norms)
+        A = res.mask.astype(bool)
+        cand = np.array([bool(rec[b]) and (res.risk[b] > 1 or lock_prev[b] > 0) for b in range(U)])
+        assert not np.any(A & ~cand)                               # A_t within C_t
+        assert np.all(A[cand & prev_active])                       # retained
+        new = cand & ~prev_active
+        admitted = np.nonzero(A & new)[0]
+        assert len(admitted) == min(max_o, int(new.sum()))         # |S_t| <= maxO, filled
+        rest = [b for b in np.nonzero(new)[0] if b not in admitted]
+        if len(admitted) and rest:                                 # the best new ones by R
+            worst = min(admitted, key=lambda b: (res.risk[b], -b))
+            best_rest = max(rest, key=lambda b: (res.risk[b], -b))
+            assert (res.risk[worst], -worst) > (res.risk[best_rest], -best_rest)
+        assert res.n_selected == int(A.sum())
+        prev_active = A
+        lock_prev = res.lock.copy()
+
+
+def test_forced_and_static_policies():
+    rng = np.random.default_rng(17)
+    U, T = 20, 25
+    rec = (rng.random(U) < 0.7).astype(np.uint8)
+    tr = _spiky_trace(rng, T, U, spike_p=0.2)
+    base = oracle.Controller(U, 3, 4, 2, recoverable=rec)
+    forced = oracle.Controller(U, 3, 4, 2, recoverable=rec, forced_recovery_steps=5)
+    stat = oracle.Controller(U, 3, 4, 2, recoverable=rec, policy=oracle.POLICY_STATIC_TOP,
+                             static_warmup_steps=6, static_fraction=0.3)
+    gsum = np.zeros(U)
+    fixed = None
+    for t, norms in enumerate(tr, start=1):
+        rb, rf, rs = base.step(norms), forced.step(norms), stat.step(norms)
+        # the policies never change the statistics
+        np.testing.assert_array_equal(rb.gnmr, rf.gnmr)
+        np.testing.assert_array_equal(rb.gnmr, rs.gnmr)
+        if t <= 5:
+            assert np.array_equal(rf.mask, rec) and rf.n_selected == rec.sum()
+        if t <= 6:
+            assert np.array_equal(rs.mask, rec)
+            gsum += np.where(rec == 1, rb.gnmr, 0.0)
+        else:
+            if fixed is None:
+                k = math.ceil(0.3 * rec.sum())
+                order = sorted(np.nonzero(rec)[0], key=lambda b: (-gsum[b], b))
+                fixed = np.zeros(U, np.uint8)
+                fixed[order[:k]] = 1
+            assert np.array_equal(rs.mask, fixed)
+            assert np.all(rs.lock == 0)
