@@ -79,7 +79,36 @@ typedef struct gnmr_config {
      * any order; a unit's segments are summed in the order given. */
     int32_t num_segments;
     const int32_t *segment_unit;  /* host [num_segments] when num_segments > 0, else ignored */
+    /* Policy variants (gnmr_policy; see there).  Defaults: ACTIVE_CAP, 0, 0, 0.25. */
+    int32_t policy;
+    int64_t forced_recovery_steps; /* steps t <= this: every recoverable unit on the recovery path */
+    int64_t static_warmup_steps;   /* GNMR_POLICY_STATIC_TOP: warm-up length */
+    double static_fraction;        /* GNMR_POLICY_STATIC_TOP: fraction of B_rec fixed, in [0, 1] */
+    /* Extra saved-activation cost c_b of recovering unit b (Eq.
+     * generic-memory-bound), host [num_units], copied; NULL = no Delta M_t. */
+    const double *unit_cost;
 } gnmr_config;
+
+/* Recovery policies.
+ *   GNMR_POLICY_ACTIVE_CAP (default): Algorithm 2, |A_t| <= maxO.
+ *   GNMR_POLICY_ADMISSION_CAP: only newly admitted units are capped (the
+ *     paper's Remark on the maxO budget): candidates that were on the
+ *     recovery path at t - 1 stay; of the other candidates at most maxO, those
+ *     with the largest R (ties: lower index), are admitted.  |A_t| can exceed
+ *     maxO and is what counts[1] reports.
+ *   GNMR_POLICY_STATIC_TOP: the ADAPT-style static baseline (App. E.4): for
+ *     t <= static_warmup_steps every recoverable unit is on the recovery path
+ *     and its GNMR is summed; at t = static_warmup_steps + 1 the
+ *     ceil(static_fraction * |B_rec|) units with the largest sum (ties: lower
+ *     index) are fixed on the recovery path for good.
+ * Independently, forced_recovery_steps (App. E.7) puts every recoverable
+ * unit on the recovery path for t <= forced_recovery_steps, with no candidate
+ * pool (statistics still update, locks are left as they are). */
+typedef enum gnmr_policy {
+    GNMR_POLICY_ACTIVE_CAP = 0,
+    GNMR_POLICY_ADMISSION_CAP = 1,
+    GNMR_POLICY_STATIC_TOP = 2
+} gnmr_policy;
 
 /* Optional per-step statistics: caller-owned DEVICE buffers.  Any pointer
  * may be NULL, and the whole struct may be NULL. */
@@ -89,7 +118,8 @@ typedef struct gnmr_stats {
     double *dgnmr;    /* [num_units] Delta-GNMR_{b,t} */
     double *risk;     /* [num_units] R_{b,t} (also reported for non-recoverable units) */
     int32_t *lock;    /* [num_units] Lock_b after the step */
-    int32_t *counts;  /* [2]: |C_t|, |A_t| */
+    int32_t *counts;  /* [2]: |C_t|, |A_t| (under STATIC_TOP: the ranked pool, the fixed set) */
+    double *delta_mem;/* [1]: Delta M_t = sum of c_b over A_t (needs unit_cost) */
 } gnmr_stats;
 
 /* Launch geometry and memory of a handle, for reporting. */
@@ -175,9 +205,10 @@ gnmr_status gnmr_finish(gnmr_handle *h, const double *d_sumsq, void *stream, uin
                         const gnmr_stats *stats);
 
 /* Checkpoint: copies the controller state (step counter t, and per unit A_b,
- * k_b, Lock_b and the GNMR window Q_b) into host_buf as a self-describing
- * blob ("GNMR", version 1, num_units, window, t, then the per-unit records and
- * windows; little-endian).  *state_bytes (if not NULL) receives the blob size;
+ * k_b, Lock_b, the active flag, the static policy's GNMR sum and the GNMR
+ * window Q_b) into host_buf as a self-describing blob ("GNMR", version 2,
+ * num_units, window, t, then the per-unit records and windows;
+ * little-endian).  *state_bytes (if not NULL) receives the blob size;
  * with host_buf == NULL nothing else happens.  Waits for `stream` (work
  * enqueued on it before the call is included), then returns.  Errors:
  * GNMR_ERR_INVALID_ARG (buf_bytes too small), GNMR_ERR_STATE, GNMR_ERR_CUDA. */

@@ -77,6 +77,8 @@ def _load():
     lib.oracle_ctl_set_policy.restype = ctypes.c_int
     lib.oracle_ctl_get_policy_state.argtypes = [P, P, P]
     lib.oracle_ctl_get_policy_state.restype = None
+    lib.oracle_ctl_set_policy_state.argtypes = [P, P, P]
+    lib.oracle_ctl_set_policy_state.restype = None
     lib.oracle_delta_mem.argtypes = [P, P, ctypes.c_int32]
     lib.oracle_delta_mem.restype = ctypes.c_double
     lib.oracle_ctl_get_state.argtypes = [P, P, P, P, P, P, P]
@@ -294,6 +296,11 @@ class Controller:
         gsum = np.empty(self.num_units, np.float64)
         _load().oracle_ctl_get_policy_state(self._h, _ptr(active), _ptr(gsum))
         return dict(active=active, gsum=gsum)
+
+    def set_policy_state(self, st: dict) -> None:
+        active = np.ascontiguousarray(st["active"], np.uint8)
+        gsum = np.ascontiguousarray(st["gsum"], np.float64)
+        _load().oracle_ctl_set_policy_state(self._h, _ptr(active), _ptr(gsum))
 
     def set_state(self, st: dict) -> None:
         A = np.ascontiguousarray(st["A"], np.float64)

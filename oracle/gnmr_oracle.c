@@ -574,6 +574,12 @@ void oracle_ctl_get_policy_state(const oracle_ctl *c, uint8_t *active, double *g
     memcpy(gsum, c->gsum, (size_t)c->num_units * sizeof(double));
 }
 
+void oracle_ctl_set_policy_state(oracle_ctl *c, const uint8_t *active, const double *gsum)
+{
+    memcpy(c->active, active, (size_t)c->num_units);
+    memcpy(c->gsum, gsum, (size_t)c->num_units * sizeof(double));
+}
+
 /* Eq. generic-memory-bound: Delta M_t = sum over b in A_t of c_b, summed in
  * unit order. */
 double oracle_delta_mem(const uint8_t *mask, const double *cost, int32_t num_units)

@@ -23,6 +23,8 @@ GNMR_DTYPE_BF16 = 1
 
 GNMR_FQ_NONE, GNMR_FQ_E2M1, GNMR_FQ_E3M2, GNMR_FQ_E4M3, GNMR_FQ_E5M2 = 0, 1, 2, 3, 4
 
+GNMR_POLICY_ACTIVE_CAP, GNMR_POLICY_ADMISSION_CAP, GNMR_POLICY_STATIC_TOP = 0, 1, 2
+
 _P = ctypes.c_void_p
 
 
@@ -45,6 +47,11 @@ class gnmr_config(ctypes.Structure):
         ("device", ctypes.c_int32),
         ("num_segments", ctypes.c_int32),
         ("segment_unit", _P),
+        ("policy", ctypes.c_int32),
+        ("forced_recovery_steps", ctypes.c_int64),
+        ("static_warmup_steps", ctypes.c_int64),
+        ("static_fraction", ctypes.c_double),
+        ("unit_cost", _P),
     ]
 
 
@@ -56,6 +63,7 @@ class gnmr_stats(ctypes.Structure):
         ("risk", _P),
         ("lock", _P),
         ("counts", _P),
+        ("delta_mem", _P),
     ]
 
 

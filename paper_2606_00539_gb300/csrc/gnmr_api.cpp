@@ -119,6 +119,8 @@ void gnmr_config_defaults(gnmr_config *cfg)
     cfg->warmup_steps = 0;
     cfg->eps = 1e-8;
     cfg->device = 0;
+    cfg->policy = GNMR_POLICY_ACTIVE_CAP;
+    cfg->static_fraction = 0.25;
 }
 
 const char *gnmr_status_string(gnmr_status s)
@@ -188,6 +190,14 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         return fail_create(GNMR_ERR_INVALID_ARG, "thresholds alpha/beta must be finite and > 0");
     if (!std::isfinite(c.eps) || c.eps < 0.0)
         return fail_create(GNMR_ERR_INVALID_ARG, "eps must be finite and >= 0");
+    if (c.policy < GNMR_POLICY_ACTIVE_CAP || c.policy > GNMR_POLICY_STATIC_TOP || c.forced_recovery_steps < 0 ||
+        c.static_warmup_steps < 0 || !(c.static_fraction >= 0.0 && c.static_fraction <= 1.0))
+        return fail_create(GNMR_ERR_INVALID_ARG,
+                           "policy, forced_recovery_steps, static_warmup_steps or static_fraction out of range");
+    if (c.unit_cost)
+        for (int32_t b = 0; b < c.num_units; ++b)
+            if (!std::isfinite(c.unit_cost[b]))
+                return fail_create(GNMR_ERR_INVALID_ARG, format("unit_cost[%d] is not finite", b));
     if (c.num_segments < 0 || (c.num_segments > 0 && !c.segment_unit))
         return fail_create(GNMR_ERR_INVALID_ARG, "num_segments must be >= 0, with segment_unit when > 0");
     const int eb = c.dtype == GNMR_DTYPE_BF16 ? 2 : 4;
@@ -287,14 +297,20 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         const size_t o_queue = cv.take(sizeof(double) * U * c.window);
         const size_t o_cand = cv.take(sizeof(gnmr::Candidate) * U);
         const size_t o_ctl = cv.take(sizeof(gnmr::Control));
+        const size_t o_cost = c.unit_cost ? cv.take(sizeof(double) * U) : 0;
 
         // Host image of the whole block: static tables plus zeroed state.
         std::vector<unsigned char> img(cv.size, 0);
         std::memcpy(&img[o_off], seg_off.data(), sizeof(int64_t) * S);
         std::memcpy(&img[o_len], seg_len.data(), sizeof(int64_t) * S);
         std::memcpy(&img[o_segu], seg_unit.data(), sizeof(int32_t) * S);
-        for (int64_t b = 0; b < U; ++b)
+        int32_t num_rec = 0;
+        for (int64_t b = 0; b < U; ++b) {
             img[o_rec + b] = c.recoverable ? (c.recoverable[b] != 0) : 1;
+            num_rec += img[o_rec + b];
+        }
+        if (c.unit_cost)
+            std::memcpy(&img[o_cost], c.unit_cost, sizeof(double) * U);
         std::memcpy(&img[o_run_seg], plan.run_seg.data(), sizeof(int64_t) * (W + 1));
         std::memcpy(&img[o_run_pos], plan.run_pos.data(), sizeof(int64_t) * (W + 1));
         std::memcpy(&img[o_first], plan.first_warp.data(), sizeof(int32_t) * U);
@@ -332,6 +348,12 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         p.queue = reinterpret_cast<double *>(base + o_queue);
         p.cand = reinterpret_cast<gnmr::Candidate *>(base + o_cand);
         p.ctl = reinterpret_cast<gnmr::Control *>(base + o_ctl);
+        p.unit_cost = c.unit_cost ? reinterpret_cast<const double *>(base + o_cost) : nullptr;
+        p.policy = c.policy;
+        p.num_recoverable = num_rec;
+        p.forced_steps = c.forced_recovery_steps;
+        p.static_warmup = c.static_warmup_steps;
+        p.static_keep = static_cast<int32_t>(std::min<double>(std::ceil(c.static_fraction * num_rec), num_rec));
         p.num_units = c.num_units;
         p.num_warps = plan.num_warps;
         p.window = c.window;
@@ -349,6 +371,7 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         h->cfg.lengths = nullptr;
         h->cfg.recoverable = nullptr;
         h->cfg.segment_unit = nullptr;
+        h->cfg.unit_cost = nullptr;
         h->num_segments = S;
         h->num_units = c.num_units;
         h->elem_bytes = eb;
@@ -405,6 +428,7 @@ gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems, 
         p.out_risk = stats->risk;
         p.out_lock = stats->lock;
         p.out_counts = stats->counts;
+        p.out_delta_mem = stats->delta_mem;
     }
     p.alpha_override = h->alpha_override;
     p.beta_override = h->beta_override;
@@ -474,6 +498,7 @@ gnmr_status gnmr_finish(gnmr_handle *h, const double *d_sumsq, void *stream, uin
         p.out_risk = stats->risk;
         p.out_lock = stats->lock;
         p.out_counts = stats->counts;
+        p.out_delta_mem = stats->delta_mem;
     }
     p.alpha_override = h->alpha_override;
     p.beta_override = h->beta_override;
@@ -529,7 +554,7 @@ gnmr_status gnmr_get_state(gnmr_handle *h, void *stream, void *host_buf, int64_t
         return fail(h, GNMR_ERR_CUDA, format("state copy: %s", cudaGetErrorString(e)));
     gnmr::StateHeader hdr{};
     std::memcpy(hdr.magic, "GNMR", 4);
-    hdr.version = 1;
+    hdr.version = 2;
     hdr.num_units = h->num_units;
     hdr.window = h->cfg.window;
     hdr.steps = ctl.steps;
@@ -546,7 +571,7 @@ gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, i
         return fail(h, GNMR_ERR_INVALID_ARG, format("state needs %lld bytes", (long long)need));
     gnmr::StateHeader hdr{};
     std::memcpy(&hdr, host_buf, sizeof hdr);
-    if (std::memcmp(hdr.magic, "GNMR", 4) != 0 || hdr.version != 1)
+    if (std::memcmp(hdr.magic, "GNMR", 4) != 0 || hdr.version != 2)
         return fail(h, GNMR_ERR_INVALID_ARG, "not a GNMR state blob (magic/version)");
     if (hdr.num_units != h->num_units || hdr.window != h->cfg.window || hdr.steps < 0)
         return fail(h, GNMR_ERR_INVALID_ARG,
@@ -559,7 +584,7 @@ gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, i
         gnmr::UnitState u;
         std::memcpy(&u, in + sizeof hdr + sizeof u * b, sizeof u);
         if (u.count < 0 || u.fill < 0 || u.fill > h->cfg.window || u.head < 0 || u.head >= h->cfg.window ||
-            u.lock < 0 || u.lock > h->cfg.lock_len)
+            u.lock < 0 || u.lock > h->cfg.lock_len || (u.active != 0 && u.active != 1))
             return fail(h, GNMR_ERR_INVALID_ARG, format("state of unit %d is out of range", b));
     }
     if (h->broken)

@@ -23,23 +23,25 @@ constexpr int64_t kUnitCostBytes = 4096;
 constexpr int64_t kSplitBytes = 512;
 constexpr int64_t kMinRunBytes = 16384;
 
-// Persistent per-unit controller state (Algorithm 1 and 2), 32 bytes.
+// Persistent per-unit controller state (Algorithm 1 and 2), 40 bytes.
 struct UnitState {
     double mean;      // A_b, historical mean of n_b
     int64_t count;    // k_b, steps at which b was observed
     int32_t fill;     // |Q_b|, valid entries of the GNMR queue (<= window)
     int32_t head;     // ring position of the oldest queue entry once full
     int32_t lock;     // Lock_b
-    int32_t pad;
+    int32_t active;   // 1 if b was on the recovery path at the previous step
+    double gsum;      // GNMR summed over the static policy's warm-up
 };
 
 // Candidate-pool entry written by the unit epilogue, read by the selection
 // (one 16-byte load).
 struct Candidate {
-    double risk;      // R_{b,t}
+    double risk;      // R_{b,t} (the static policy ranks by the GNMR sum)
     int32_t unit;
-    int32_t lock;     // Lock_b before this step
+    uint32_t lock;    // Lock_b before this step, bit 31: active at the previous step
 };
+constexpr uint32_t kCandActive = 0x80000000u;
 
 // Device-resident step control block.
 struct Control {
@@ -52,7 +54,7 @@ struct Control {
 // buffers double[num_units * window] (little-endian, as on the device).
 struct StateHeader {
     char magic[4];        // "GNMR"
-    uint32_t version;     // 1
+    uint32_t version;     // 2
     int32_t num_units;
     int32_t window;
     int64_t steps;
@@ -81,6 +83,14 @@ struct StepParams {
     int32_t *out_lock, *out_counts;                       // caller, optional
     double *out_sumsq;                                    // kStepPartials output [U]
     const double *in_sumsq;                               // kStepFinish input [U]
+    double *out_delta_mem;                                // caller, optional [1]
+    const double *unit_cost;                              // [U] or null
+    int32_t policy;
+    int32_t num_recoverable;
+    int64_t forced_steps;
+    int64_t static_warmup;
+    int32_t static_keep;                                  // ceil(static_fraction * |B_rec|)
+    int32_t pad2;
     int32_t num_units;
     int32_t num_warps;
     int32_t window;

@@ -209,11 +209,11 @@ __device__ __forceinline__ double pick_threshold(double override_value, int64_t 
 // about one memory round trip; candidates are appended with one atomic per
 // warp.  Called by all 32 lanes.
 __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, double sumsq,
-                              double alpha, double beta)
+                              double alpha, double beta, int64_t t)
 {
     bool cand = false;
     double r = 0.0;
-    int32_t lock_prev = 0;
+    uint32_t cand_lock = 0;
     if (active) {
         const double n = sqrt(sumsq);
         UnitState s = p.state[b];
@@ -273,13 +273,35 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
         if (p.out_dgnmr) p.out_dgnmr[b] = d;
         if (p.out_risk) p.out_risk[b] = r;
 
-        lock_prev = s.lock;
-        cand = p.recoverable[b] && (r > 1.0 || s.lock > 0);
-        if (!cand) {
-            // Not a candidate: Lock_b is already 0 and b stays on the low-cost path.
-            p.mask[b] = 0;
-            if (p.out_lock) p.out_lock[b] = 0;
+        const bool rec = p.recoverable[b] != 0;
+        const bool stat = p.policy == 2;
+        if (stat && t <= p.static_warmup && rec)
+            p.state[b].gsum = s.gsum + g;
+        if (t <= p.forced_steps || (stat && t <= p.static_warmup)) {
+            // every recoverable unit on the recovery path; locks untouched
+            p.mask[b] = rec ? 1 : 0;
+            p.state[b].active = rec ? 1 : 0;
+            if (p.out_lock) p.out_lock[b] = s.lock;
+        } else if (stat) {
+            if (t == p.static_warmup + 1 && rec) {
+                cand = true;                          // ranked once by the warm-up's GNMR sum
+                r = s.gsum;
+            } else {
+                p.mask[b] = (rec && t > p.static_warmup + 1 && s.active) ? 1 : 0;
+                if (t == p.static_warmup + 1)
+                    p.state[b].active = 0;
+                if (p.out_lock) p.out_lock[b] = s.lock;
+            }
+        } else {
+            cand = rec && (r > 1.0 || s.lock > 0);
+            if (!cand) {
+                // Not a candidate: Lock_b is already 0 and b stays on the low-cost path.
+                p.mask[b] = 0;
+                p.state[b].active = 0;
+                if (p.out_lock) p.out_lock[b] = 0;
+            }
         }
+        cand_lock = static_cast<uint32_t>(s.lock) | (s.active ? kCandActive : 0u);
     }
     const unsigned want = __ballot_sync(kFull, cand);
     if (want) {
@@ -294,7 +316,7 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
             if (slot < static_cast<uint32_t>(p.num_units)) {   // at most one entry per unit
                 p.cand[slot].risk = r;
                 p.cand[slot].unit = b;
-                p.cand[slot].lock = lock_prev;
+                p.cand[slot].lock = cand_lock;
             }
         }
     }
@@ -337,20 +359,21 @@ __device__ __forceinline__ uint32_t index_key(int32_t b, int32_t num_units)
     return static_cast<uint32_t>(num_units - 1 - b);
 }
 
-__device__ __forceinline__ void load_candidate(const Candidate *c, double &r, int32_t &b, int32_t &lock)
+__device__ __forceinline__ void load_candidate(const Candidate *c, double &r, int32_t &b, uint32_t &lock)
 {
     const double2 v = __ldcg(reinterpret_cast<const double2 *>(c));
     const uint64_t w = static_cast<uint64_t>(__double_as_longlong(v.y));
     r = v.x;
     b = static_cast<int32_t>(w & 0xffffffffu);
-    lock = static_cast<int32_t>(w >> 32);
+    lock = static_cast<uint32_t>(w >> 32);
 }
 
-// K-th largest 96-bit key (risk_key : index_key) among the m candidates,
-// 1 <= K < m, by most-significant-digit radix select with 8-bit digits.
+// K-th largest 96-bit key (risk_key : index_key) among the m candidates (or
+// among those not active at t-1 when only_new), 1 <= K < that count, by
+// most-significant-digit radix select with 8-bit digits.
 // Returns the threshold: exactly K keys compare >= it.  All threads of the
 // CTA call this.
-__device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, uint32_t *hist,
+__device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, bool only_new, uint32_t *hist,
                              uint32_t *misc, uint64_t &thr_hi, uint32_t &thr_lo)
 {
     const int lo_bits = p.num_units > 1 ? 32 - __clz(static_cast<uint32_t>(p.num_units - 1)) : 0;
@@ -366,7 +389,8 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, uint32
         __syncthreads();
         for (uint32_t i0 = threadIdx.x; i0 < m; i0 += 4 * blockDim.x) {
             double rr[4];
-            int32_t bb[4], ll[4];
+            int32_t bb[4];
+            uint32_t ll[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {           // four loads in flight per thread
                 const uint32_t i = i0 + j * blockDim.x;
@@ -377,6 +401,8 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, uint32
             for (int j = 0; j < 4; ++j) {
                 if (i0 + j * blockDim.x >= m)
                     break;
+                if (only_new && (ll[j] & kCandActive))
+                    continue;
                 const uint64_t hi = risk_key(rr[j]);
                 const uint32_t lo = index_key(bb[j], p.num_units);
                 if ((hi & msk_hi) == pre_hi && (lo & msk_lo) == pre_lo) {
@@ -436,39 +462,111 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, uint32
     thr_lo = pre_lo;
 }
 
-// Last CTA: Top_maxO, Algorithm 2's lock bookkeeping, mask, counts, reset.
-__device__ void select_and_commit(const StepParams &p, uint32_t *hist, uint32_t *misc)
+// Block-wide sum of per-thread counts (all threads get it).
+__device__ __forceinline__ uint32_t block_count(uint32_t v, uint32_t *slot)
+{
+    if (threadIdx.x == 0)
+        *slot = 0;
+    __syncthreads();
+    v = __reduce_add_sync(kFull, v);
+    if ((threadIdx.x & 31) == 0 && v)
+        atomicAdd(slot, v);
+    __syncthreads();
+    return *slot;
+}
+
+// Delta M_t = sum of c_b over the units on the recovery path, in a fixed
+// order (thread-strided partial sums, then a fixed tree), so the value is
+// reproducible run to run.
+__device__ void delta_mem(const StepParams &p, double *red)
+{
+    double acc = 0.0;
+    for (int32_t b = threadIdx.x; b < p.num_units; b += blockDim.x)
+        if (__ldcg(p.mask + b))
+            acc += p.unit_cost[b];
+    red[threadIdx.x] = acc;
+    __syncthreads();
+    for (unsigned o = blockDim.x / 2; o > 0; o >>= 1) {
+        if (threadIdx.x < o)
+            red[threadIdx.x] += red[threadIdx.x + o];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0)
+        *p.out_delta_mem = red[0];
+}
+
+// Last CTA: Top_maxO (or the policy's choice), Algorithm 2's lock
+// bookkeeping, mask, counts, Delta M_t, reset.
+__device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist, uint32_t *misc, double *red)
 {
     uint32_t m = __ldcg(&p.ctl->n_cand);
     m = m < static_cast<uint32_t>(p.num_units) ? m : static_cast<uint32_t>(p.num_units);
-    const uint32_t cap = static_cast<uint32_t>(p.max_o);
-    const uint32_t K = m < cap ? m : cap;
-    const bool take_all = m <= cap;
-    uint64_t thr_hi = 0;
-    uint32_t thr_lo = 0;
-    if (!take_all && K > 0)
-        radix_select(p, m, K, hist, misc, thr_hi, thr_lo);
-    for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
-        double r;
-        int32_t b, prev;
-        load_candidate(p.cand + i, r, b, prev);
-        bool sel;
-        if (take_all) {
-            sel = true;
-        } else if (K == 0) {
-            sel = false;
-        } else {
-            const uint64_t hi = risk_key(r);
-            sel = hi > thr_hi || (hi == thr_hi && index_key(b, p.num_units) >= thr_lo);
+    const bool all_on = t <= p.forced_steps || (p.policy == 2 && t <= p.static_warmup);
+    const bool stat = p.policy == 2 && !all_on;
+    const bool admission = p.policy == 1 && !all_on;
+    uint32_t n_sel = 0;
+    if (all_on) {
+        m = 0;
+        n_sel = static_cast<uint32_t>(p.num_recoverable);
+    } else if (stat && t > p.static_warmup + 1) {
+        m = 0;
+        n_sel = static_cast<uint32_t>(p.static_keep);
+    } else {
+        // the pool the cap applies to: every candidate, or the new ones only
+        uint32_t pool = m;
+        uint32_t retained = 0;
+        if (admission) {
+            uint32_t mine = 0;
+            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x)
+                mine += (__ldcg(&p.cand[i].lock) & kCandActive) ? 1u : 0u;
+            retained = block_count(mine, &misc[4]);     // misc[0] holds the last-CTA flag
+            pool = m - retained;
         }
-        const int32_t next = !sel ? 0 : (r > 1.0 ? p.lock_len : (prev - 1 > 0 ? prev - 1 : 0));
-        p.state[b].lock = next;
-        p.mask[b] = sel ? 1 : 0;
-        if (p.out_lock) p.out_lock[b] = next;
+        const uint32_t cap = stat ? static_cast<uint32_t>(p.static_keep) : static_cast<uint32_t>(p.max_o);
+        const uint32_t K = pool < cap ? pool : cap;
+        const bool take_all = pool <= cap;
+        uint64_t thr_hi = 0;
+        uint32_t thr_lo = 0;
+        if (!take_all && K > 0)
+            radix_select(p, m, K, admission, hist, misc, thr_hi, thr_lo);
+        for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+            double r;
+            int32_t b;
+            uint32_t lk;
+            load_candidate(p.cand + i, r, b, lk);
+            const bool was_active = (lk & kCandActive) != 0;
+            const int32_t prev = static_cast<int32_t>(lk & ~kCandActive);
+            bool sel;
+            if (admission && was_active) {
+                sel = true;                              // retained without counting against the cap
+            } else if (take_all) {
+                sel = true;
+            } else if (K == 0) {
+                sel = false;
+            } else {
+                const uint64_t hi = risk_key(r);
+                sel = hi > thr_hi || (hi == thr_hi && index_key(b, p.num_units) >= thr_lo);
+            }
+            int32_t next;
+            if (stat)
+                next = prev;                             // the static policy keeps no locks
+            else
+                next = !sel ? 0 : (r > 1.0 ? p.lock_len : (prev - 1 > 0 ? prev - 1 : 0));
+            p.state[b].lock = next;
+            p.state[b].active = sel ? 1 : 0;
+            p.mask[b] = sel ? 1 : 0;
+            if (p.out_lock) p.out_lock[b] = next;
+        }
+        n_sel = K + retained;
     }
     if (threadIdx.x == 0 && p.out_counts) {
         p.out_counts[0] = static_cast<int32_t>(m);
-        p.out_counts[1] = static_cast<int32_t>(K);
+        p.out_counts[1] = static_cast<int32_t>(n_sel);
+    }
+    __syncthreads();
+    if (p.unit_cost && p.out_delta_mem) {
+        __threadfence_block();
+        delta_mem(p, red);
     }
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -487,7 +585,8 @@ __global__ void __launch_bounds__(kThreads, kMinCtasPerSm)
 gnmr_step_kernel(const __grid_constant__ StepParams p)
 {
     __shared__ uint32_t s_hist[256];
-    __shared__ uint32_t s_misc[4];
+    __shared__ uint32_t s_misc[8];
+    __shared__ double s_red[kThreads];
     constexpr int kEB = Elem<DT>::kBytes;
     const int lane = threadIdx.x & 31;
     const int warp = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
@@ -501,7 +600,7 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
             const int64_t b = b0 + lane;
             const bool active = b < p.num_units;
             const double s = active ? p.in_sumsq[b] : 0.0;
-            unit_epilogue(p, active, active ? static_cast<int32_t>(b) : 0, s, alpha, beta);
+            unit_epilogue(p, active, active ? static_cast<int32_t>(b) : 0, s, alpha, beta, t);
         }
     } else if (warp < p.num_warps) {
         // t, alpha_t and beta_t are fixed for the whole step.
@@ -534,7 +633,7 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
                         pend_s = s;
                     }
                     if (++npend == 32) {
-                        unit_epilogue(p, true, pend_b, pend_s, alpha, beta);
+                        unit_epilogue(p, true, pend_b, pend_s, alpha, beta, t);
                         npend = 0;
                     }
                 }
@@ -565,7 +664,7 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
         if (cur >= 0)
             complete(cur, cur_s);
         if (MODE != kStepPartials && npend > 0)
-            unit_epilogue(p, lane < npend, pend_b, pend_s, alpha, beta);
+            unit_epilogue(p, lane < npend, pend_b, pend_s, alpha, beta, t);
     }
     if (MODE == kStepPartials)
         return;
@@ -578,7 +677,7 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     __syncthreads();
     if (s_misc[0]) {
         __threadfence();
-        select_and_commit(p, s_hist, s_misc);
+        select_and_commit(p, __ldcg(&p.ctl->steps) + 1, s_hist, s_misc, s_red);
     }
 }
 

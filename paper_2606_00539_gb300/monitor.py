@@ -27,11 +27,15 @@ class Monitor:
     recoverable: per-unit flags (B_rec); None = every unit recoverable.
     alpha, beta: (init, main) thresholds; the init values hold for steps
     t <= warmup_steps (two-stage schedule).  A scalar means both stages.
+    policy, forced_recovery_steps, static_warmup_steps, static_fraction: the
+    recovery policy variants of include/gnmr.h; unit_cost: per-unit c_b for
+    the Delta M_t statistic.
     """
 
     def __init__(self, offsets, lengths, *, dtype="bf16", recoverable=None, window=8, max_o=4,
                  lock_len=1, alpha=(1.5, 1.1), beta=(1.5, 1.5), warmup_steps=0, eps=1e-8,
-                 device=0, segment_unit=None, num_units=None):
+                 device=0, segment_unit=None, num_units=None, policy=0, forced_recovery_steps=0,
+                 static_warmup_steps=0, static_fraction=0.25, unit_cost=None):
         self._h = None
         off = np.ascontiguousarray(offsets, dtype=np.int64)
         ln = np.ascontiguousarray(lengths, dtype=np.int64)
@@ -75,6 +79,16 @@ class Monitor:
         cfg.warmup_steps = int(warmup_steps)
         cfg.eps = float(eps)
         cfg.device = int(device.index if hasattr(device, "index") else device)
+        cfg.policy = int(policy)
+        cfg.forced_recovery_steps = int(forced_recovery_steps)
+        cfg.static_warmup_steps = int(static_warmup_steps)
+        cfg.static_fraction = float(static_fraction)
+        cost = None
+        if unit_cost is not None:
+            cost = np.ascontiguousarray(unit_cost, dtype=np.float64)
+            if cost.shape != (U,):
+                raise ValueError("unit_cost must have one entry per unit")
+            cfg.unit_cost = cost.ctypes.data
         self._h = N.gnmr_create(cfg)
         self.num_units = U
         self.dtype = cfg.dtype
@@ -118,6 +132,7 @@ class Monitor:
             "risk": torch.empty(U, dtype=torch.float64, device=dev),
             "lock": torch.empty(U, dtype=torch.int32, device=dev),
             "counts": torch.empty(2, dtype=torch.int32, device=dev),
+            "delta_mem": torch.zeros(1, dtype=torch.float64, device=dev),
         }
 
     def _check_tensor(self, t, name, dtype, numel=None):
@@ -141,7 +156,8 @@ class Monitor:
                            ("dgnmr", torch.float64, self.num_units),
                            ("risk", torch.float64, self.num_units),
                            ("lock", torch.int32, self.num_units),
-                           ("counts", torch.int32, 2)):
+                           ("counts", torch.int32, 2),
+                           ("delta_mem", torch.float64, 1)):
             if stats.get(key) is not None:
                 self._check_tensor(stats[key], key, dt, n)
                 setattr(st, key, stats[key].data_ptr())

@@ -61,9 +61,11 @@ int main(void) {
   F(gnmr_config, max_o) F(gnmr_config, lock_len) F(gnmr_config, alpha_init)
   F(gnmr_config, alpha_main) F(gnmr_config, beta_init) F(gnmr_config, beta_main)
   F(gnmr_config, warmup_steps) F(gnmr_config, eps) F(gnmr_config, device)
-  F(gnmr_config, num_segments) F(gnmr_config, segment_unit)
+  F(gnmr_config, num_segments) F(gnmr_config, segment_unit) F(gnmr_config, policy)
+  F(gnmr_config, forced_recovery_steps) F(gnmr_config, static_warmup_steps)
+  F(gnmr_config, static_fraction) F(gnmr_config, unit_cost)
   F(gnmr_stats, norm) F(gnmr_stats, gnmr) F(gnmr_stats, dgnmr) F(gnmr_stats, risk)
-  F(gnmr_stats, lock) F(gnmr_stats, counts)
+  F(gnmr_stats, lock) F(gnmr_stats, counts) F(gnmr_stats, delta_mem)
   F(gnmr_info, num_units) F(gnmr_info, dtype) F(gnmr_info, device) F(gnmr_info, num_ctas)
   F(gnmr_info, threads_per_cta) F(gnmr_info, num_warps) F(gnmr_info, num_partials)
   F(gnmr_info, device_bytes) F(gnmr_info, arena_elems_min) F(gnmr_info, steps)
@@ -107,7 +109,8 @@ def _valid_cfg(off, ln):
 @pytest.mark.parametrize("field,value", [
     ("num_units", 0), ("dtype", 7), ("window", 0), ("max_o", -1), ("lock_len", -1),
     ("alpha_init", 0.0), ("alpha_main", float("inf")), ("beta_init", -1.0),
-    ("beta_main", float("nan")), ("eps", -1e-3), ("warmup_steps", -5),
+    ("beta_main", float("nan")), ("eps", -1e-3), ("warmup_steps", -5), ("policy", 3),
+    ("forced_recovery_steps", -1), ("static_fraction", 1.5), ("static_warmup_steps", -2),
 ])
 def test_create_rejects_bad_config_before_cuda(lib, field, value):
     off = np.array([0, 10], np.int64)

@@ -27,6 +27,13 @@ def _monitor(w, **over):
     return Monitor(w.offsets, w.lengths, device=0, **kw)
 
 
+def _policy_kwargs(cfg):
+    from fractions import Fraction
+    return dict(policy=int(cfg.get("policy", 0)), forced_recovery_steps=int(cfg.get("forced", 0)),
+                static_warmup_steps=int(cfg.get("static_warmup", 0)),
+                static_fraction=float(cfg.get("static_fraction", Fraction(1, 4))))
+
+
 def _run_lockstep(w, steps=None, every=1):
     tr = TD.LockstepTrace(w, "cuda:0", _monitor)
     try:
@@ -120,7 +127,8 @@ def test_hand_trace_on_gpu(trace, cuda_device):
                   lock_len=int(cfg["lock_len"]),
                   alpha=(float(cfg["alpha_init"]), float(cfg["alpha_main"])),
                   beta=(float(cfg["beta_init"]), float(cfg["beta_main"])),
-                  warmup_steps=int(cfg["warmup"]), eps=float(cfg["eps"]), device=0)
+                  warmup_steps=int(cfg["warmup"]), eps=float(cfg["eps"]), device=0,
+                  **_policy_kwargs(cfg))
     stats = mon.new_stats()
     arena = torch.zeros(4 * U, dtype=torch.float32, device=cuda_device)
     try:

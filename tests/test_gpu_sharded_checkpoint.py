@@ -67,11 +67,12 @@ def test_sharded_step_matches_oracle(config, shrink, world, cuda_device):
 
 def _parse_blob(blob, U, window):
     magic, version, nu, win, steps, _ = struct.unpack_from("<4sIiiqq", blob, 0)
-    assert magic == b"GNMR" and version == 1 and nu == U and win == window
+    assert magic == b"GNMR" and version == 2 and nu == U and win == window
     rec = np.frombuffer(blob, dtype=np.dtype([("A", "<f8"), ("k", "<i8"), ("fill", "<i4"),
-                                              ("head", "<i4"), ("lock", "<i4"), ("pad", "<i4")]),
+                                              ("head", "<i4"), ("lock", "<i4"), ("active", "<i4"),
+                                              ("gsum", "<f8")]),
                         count=U, offset=32)
-    q = np.frombuffer(blob, dtype="<f8", count=U * window, offset=32 + 32 * U).reshape(U, window)
+    q = np.frombuffer(blob, dtype="<f8", count=U * window, offset=32 + 40 * U).reshape(U, window)
     return steps, rec, q
 
 
@@ -90,6 +91,7 @@ def test_checkpoint_blob_matches_oracle_state(cuda_device):
         assert np.array_equal(rec["k"], st["k"])
         assert np.array_equal(rec["fill"], st["qlen"])
         assert np.array_equal(rec["lock"], st["lock"])
+        assert np.array_equal(rec["active"], tr.ctl.policy_state()["active"])
         for b in range(w.num_units):        # ring (oldest at head) vs oldest-first list
             n = rec["fill"][b]
             ring = np.roll(q[b], -rec["head"][b])[:n] if n == w.window else q[b][:n]

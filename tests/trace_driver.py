@@ -40,15 +40,28 @@ def _exactness(state, res, w, t, alpha=math.nan, beta=math.nan):
     return exact
 
 
-def margin_violations(state_before, res, w, t, alpha=math.nan, beta=math.nan):
+def margin_violations(state_before, res, w, t, alpha=math.nan, beta=math.nan, policy=None,
+                      active_before=None):
     """Units whose GPU decision could differ from the oracle's by rounding.
-    ``w`` needs alpha, beta, warmup_steps, window, max_o and recoverable."""
+    ``w`` needs alpha, beta, warmup_steps, window, max_o and recoverable;
+    ``policy`` (dict of the policy settings) and ``active_before`` (A_{t-1})
+    for the policy variants."""
+    policy = policy or {}
+    forced = policy.get("forced_recovery_steps", 0)
+    kind = policy.get("policy", 0)
+    warm = policy.get("static_warmup_steps", 0)
+    if t <= forced or (kind == 2 and t <= warm):
+        return []                                   # no decision depends on a rounded value
     rec = np.asarray(w.recoverable).astype(bool)
+    if kind == 2:
+        return []                                   # the static choice is checked separately
     exact = _exactness(state_before, res, w, t, alpha, beta)
     r = res.risk
     bad = set(np.nonzero(rec & ~exact & (np.abs(r - 1.0) < MARGIN))[0].tolist())
     lock_prev = state_before["lock"]
     cand = np.nonzero(rec & ((r > 1.0) | (lock_prev > 0)))[0]
+    if kind == 1 and active_before is not None:    # the cap applies to new candidates only
+        cand = np.array([b for b in cand if not active_before[b]], dtype=np.int64)
     if len(cand) > w.max_o and w.max_o > 0:
         order = sorted(cand.tolist(), key=lambda b: (-r[b], b))
         a, b = order[w.max_o - 1], order[w.max_o]
@@ -70,15 +83,18 @@ class StepRecord:
 class LockstepTrace:
     """Drives one workload on the GPU monitor and the oracle."""
 
-    def __init__(self, w: workloads.Workload, device, monitor_factory, threads: int = 0):
+    def __init__(self, w: workloads.Workload, device, monitor_factory, threads: int = 0,
+                 policy: dict | None = None):
         import torch
         self.torch = torch
         self.w = w
         self.dev = torch.device(device)
         self.filler = workloads.Filler(w, self.dev)
         self.arena = self.filler.new_arena()
-        self.mon = monitor_factory(w)
-        self.ctl = oracle.Controller(w.num_units, **w.controller_kwargs())
+        self.policy = dict(policy or {})
+        self.mon = monitor_factory(w, **self.policy) if self.policy else monitor_factory(w)
+        ctl_policy = {k: v for k, v in self.policy.items() if k != "unit_cost"}
+        self.ctl = oracle.Controller(w.num_units, **w.controller_kwargs(), **ctl_policy)
         self.stats = self.mon.new_stats()
         self.threads = threads or min(16, os.cpu_count() or 1)
         self.records = []
@@ -130,13 +146,16 @@ class LockstepTrace:
         rec = StepRecord(t + 1, 0)
         while True:
             before = self.ctl.get_state()
+            policy_before = self.ctl.policy_state()
+            active_before = policy_before["active"]
             res = self.ctl.step(norms, alpha, beta)
-            bad = margin_violations(before, res, w, t + 1, alpha, beta)
+            bad = margin_violations(before, res, w, t + 1, alpha, beta, self.policy, active_before)
             if not bad:
                 break
             if rec.attempts >= MAX_ATTEMPTS:
                 raise RuntimeError(f"step {t + 1}: no margin after {MAX_ATTEMPTS} redraws: {bad[:8]}")
             self.ctl.set_state(before)
+            self.ctl.set_policy_state(policy_before)
             rec.attempts += 1
             segs = []
             for u in bad:                                  # one factor for all of a unit's tensors
