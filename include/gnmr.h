@@ -134,6 +134,8 @@ typedef struct gnmr_info {
     int64_t device_bytes;      /* library-owned device memory */
     int64_t arena_elems_min;   /* max over units of offset + length */
     int64_t steps;             /* gnmr_step calls enqueued so far */
+    int32_t variant;           /* streaming-loop shape: 0 many-small-units, 1 large units */
+    int32_t reserved;
 } gnmr_info;
 
 typedef struct gnmr_handle gnmr_handle;

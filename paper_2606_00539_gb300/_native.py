@@ -79,6 +79,8 @@ class gnmr_info(ctypes.Structure):
         ("device_bytes", ctypes.c_int64),
         ("arena_elems_min", ctypes.c_int64),
         ("steps", ctypes.c_int64),
+        ("variant", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
     ]
 
 

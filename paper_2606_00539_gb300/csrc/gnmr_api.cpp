@@ -22,6 +22,7 @@ struct gnmr_handle {
     int elem_bytes = 0;
     int32_t num_ctas = 0;
     int32_t finish_ctas = 0;      // grid of the controller-only launch
+    int32_t variant = 0;          // streaming-loop shape (gnmr::kVariant*)
     int32_t num_warps = 0;
     int64_t num_segments = 0;
     int64_t num_partials = 0;
@@ -227,10 +228,16 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
     if (scope.status() != cudaSuccess)
         return fail_create(GNMR_ERR_CUDA, format("cudaSetDevice(%d): %s", c.device,
                                                  cudaGetErrorString(scope.status())));
+    // the streaming-loop variant follows the mean unit size
+    int64_t grad_bytes = 0;
+    for (int64_t g = 0; g < S_in; ++g)
+        grad_bytes += c.lengths[g] * eb;
+    const int variant = grad_bytes / c.num_units >= gnmr::kBulkUnitBytes ? gnmr::kVariantBulk
+                                                                         : gnmr::kVariantSmall;
     int sms = 0, per_sm = 0;
     cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
     if (e == cudaSuccess)
-        e = gnmr::step_occupancy(c.dtype, &per_sm);
+        e = gnmr::step_occupancy(c.dtype, variant, &per_sm);
     if (e != cudaSuccess || sms < 1 || per_sm < 1)
         return fail_create(GNMR_ERR_CUDA, format("device query failed: %s", cudaGetErrorString(e)));
 
@@ -373,6 +380,7 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         h->cfg.segment_unit = nullptr;
         h->cfg.unit_cost = nullptr;
         h->num_segments = S;
+        h->variant = variant;
         h->num_units = c.num_units;
         h->elem_bytes = eb;
         h->num_warps = plan.num_warps;
@@ -432,8 +440,8 @@ gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems, 
     }
     p.alpha_override = h->alpha_override;
     p.beta_override = h->beta_override;
-    const cudaError_t e = gnmr::launch_step(p, h->cfg.dtype, h->num_ctas,
-                                            static_cast<cudaStream_t>(stream));
+    const cudaError_t e = gnmr::launch_step(p, h->cfg.dtype, h->num_ctas, static_cast<cudaStream_t>(stream),
+                                            gnmr::kStepFull, h->variant);
     if (e != cudaSuccess) {
         h->broken = true;
         return fail(h, GNMR_ERR_CUDA, format("step launch: %s", cudaGetErrorString(e)));
@@ -468,7 +476,7 @@ gnmr_status gnmr_step_partials(gnmr_handle *h, const void *d_arena, int64_t aren
     p.arena = d_arena;
     p.out_sumsq = d_sumsq;
     const cudaError_t e = gnmr::launch_step(p, h->cfg.dtype, h->num_ctas, static_cast<cudaStream_t>(stream),
-                                            gnmr::kStepPartials);
+                                            gnmr::kStepPartials, h->variant);
     if (e != cudaSuccess) {
         h->broken = true;
         return fail(h, GNMR_ERR_CUDA, format("partials launch: %s", cudaGetErrorString(e)));
@@ -638,6 +646,8 @@ gnmr_status gnmr_get_info(const gnmr_handle *h, gnmr_info *info)
     info->device_bytes = h->device_bytes;
     info->arena_elems_min = h->max_end;
     info->steps = h->steps;
+    info->variant = h->variant;
+    info->reserved = 0;
     return GNMR_OK;
 }
 

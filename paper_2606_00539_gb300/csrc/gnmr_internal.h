@@ -9,11 +9,16 @@
 
 namespace gnmr {
 
-// Launch shape of the step kernel.  512 threads = 16 warps per CTA; the
-// kernel is compiled for two resident CTAs per SM (<= 64 registers/thread).
+// Launch shape of the step kernel: 512 threads = 16 warps per CTA.  Two
+// compiled variants of the streaming loop (gnmr_kernels.cu): kVariantSmall
+// (two resident CTAs per SM) for layouts of many small units, kVariantBulk
+// (one CTA per SM, deeper per-warp streams) for layouts whose mean unit holds
+// at least kBulkUnitBytes.
 constexpr int kThreads = 512;
 constexpr int kWarpsPerCta = kThreads / 32;
-constexpr int kMinCtasPerSm = 2;
+constexpr int kVariantSmall = 0;
+constexpr int kVariantBulk = 1;
+constexpr int64_t kBulkUnitBytes = int64_t(1) << 20;
 
 // Work partition: a unit costs its element bytes plus this many bytes of
 // equivalent fixed work (reduction, Algorithm 1 update, bookkeeping); runs
@@ -110,10 +115,10 @@ constexpr int kStepFinish = 2;
 
 // Enqueues one launch of the step kernel in `mode`; returns the launch status.
 cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream,
-                        int mode = kStepFull);
+                        int mode = kStepFull, int variant = kVariantSmall);
 
-// Resident CTAs per SM of the step kernel for `dtype`.
-cudaError_t step_occupancy(int dtype, int *ctas_per_sm);
+// Resident CTAs per SM of the step kernel for `dtype` and `variant`.
+cudaError_t step_occupancy(int dtype, int variant, int *ctas_per_sm);
 
 // Records the failure detail that gnmr_last_error(NULL) reports on the
 // calling thread (used by calls that have no handle).

@@ -39,8 +39,21 @@ namespace gnmr {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kUnroll = 8;   // 16-byte loads in flight per lane
 constexpr int kFlush = 16;   // main-loop iterations summed in fp32 before the fp64 add
+
+// Two compiled shapes of the streaming loop, chosen per handle from the mean
+// unit size (measured on GB300, see the design notes): many small units run
+// best with 8 16-byte loads in flight per lane and two CTAs per SM; large
+// units with 16 loads per lane and one CTA per SM (fewer, deeper streams).
+template <int V> struct Shape;
+template <> struct Shape<kVariantSmall> {
+    static constexpr int kUnroll = 8;
+    static constexpr int kMinCtas = 2;
+};
+template <> struct Shape<kVariantBulk> {
+    static constexpr int kUnroll = 16;
+    static constexpr int kMinCtas = 1;
+};
 
 template <int DT> struct Elem;
 template <> struct Elem<0> {             // fp32
@@ -54,13 +67,36 @@ template <> struct Elem<1> {             // bf16, two per 32-bit word
 
 // 16-byte streaming load: non-coherent read-only path, no L1 allocation,
 // 256-byte L2 prefetch granularity.
-__device__ __forceinline__ uint4 ld_stream16(const uint4 *p)
+constexpr int kVecWords = 4;
+constexpr int kVecBytes = 16;
+struct alignas(kVecBytes) Vec {
+    uint32_t w[kVecWords];
+};
+
+__device__ __forceinline__ Vec ld_stream(const Vec *p)
 {
-    uint4 r;
+    Vec r;
     asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
-        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-        : "l"(p));
+        : "=r"(r.w[0]), "=r"(r.w[1]), "=r"(r.w[2]), "=r"(r.w[3]) : "l"(p));
     return r;
+}
+
+__device__ __forceinline__ Vec zero_vec()
+{
+    Vec r;
+#pragma unroll
+    for (int i = 0; i < kVecWords; ++i)
+        r.w[i] = 0u;
+    return r;
+}
+
+__device__ __forceinline__ uint32_t vec_or(const Vec &v)
+{
+    uint32_t o = 0;
+#pragma unroll
+    for (int i = 0; i < kVecWords; ++i)
+        o |= v.w[i];
+    return o;
 }
 
 // One element as an fp32 bit pattern (bf16 is the upper half of an fp32).
@@ -74,22 +110,27 @@ template <> __device__ __forceinline__ uint32_t ld_elem_bits<1>(const char *p)
     return static_cast<uint32_t>(__ldg(reinterpret_cast<const unsigned short *>(p))) << 16;
 }
 
-// Sum of squares of the elements packed in one 16-byte vector, in fp32.
-template <int DT> __device__ __forceinline__ float vec_sumsq(const uint4 v);
-template <> __device__ __forceinline__ float vec_sumsq<0>(const uint4 v)
-{
-    const float a = __uint_as_float(v.x), b = __uint_as_float(v.y);
-    const float c = __uint_as_float(v.z), d = __uint_as_float(v.w);
-    return fmaf(d, d, fmaf(c, c, fmaf(b, b, a * a)));
-}
-template <> __device__ __forceinline__ float vec_sumsq<1>(const uint4 v)
+// Sum of squares of the elements packed in one vector, in fp32 (two
+// independent chains per vector).
+template <int DT> __device__ __forceinline__ float vec_sumsq(const Vec &v);
+template <> __device__ __forceinline__ float vec_sumsq<0>(const Vec &v)
 {
     float s0 = 0.f, s1 = 0.f;
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float lo = __uint_as_float(w[i] << 16);
-        const float hi = __uint_as_float(w[i] & 0xffff0000u);
+    for (int i = 0; i < kVecWords; i += 2) {
+        const float a = __uint_as_float(v.w[i]), b = __uint_as_float(v.w[i + 1]);
+        s0 = fmaf(a, a, s0);
+        s1 = fmaf(b, b, s1);
+    }
+    return s0 + s1;
+}
+template <> __device__ __forceinline__ float vec_sumsq<1>(const Vec &v)
+{
+    float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+    for (int i = 0; i < kVecWords; ++i) {
+        const float lo = __uint_as_float(v.w[i] << 16);
+        const float hi = __uint_as_float(v.w[i] & 0xffff0000u);
         s0 = fmaf(lo, lo, s0);
         s1 = fmaf(hi, hi, s1);
     }
@@ -110,14 +151,15 @@ __device__ __forceinline__ double warp_allreduce_sum(double v)
 // in every lane and sets `suspect` when fp32 squaring may have lost accuracy:
 // a nonzero segment whose sum is below 2^-100 (denormal squares) or above
 // 2^100 (possible fp32 overflow), or a NaN/Inf sum.
-template <int DT>
+template <int DT, int kUnroll>
 __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n, int lane,
                                                      bool &suspect)
 {
     constexpr int kEB = Elem<DT>::kBytes;
-    constexpr int kVE = 16 / kEB;
-    const uint32_t mis = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(seg) & 15u);
-    int64_t head = static_cast<int64_t>(((16u - mis) & 15u) / kEB);
+    constexpr int kVE = kVecBytes / kEB;
+    constexpr uint32_t kAlign = kVecBytes - 1;
+    const uint32_t mis = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(seg) & kAlign);
+    int64_t head = static_cast<int64_t>(((kVecBytes - mis) & kAlign) / kEB);
     head = head < n ? head : n;
     const int64_t nvec = (n - head) / kVE;
     const int64_t tail = n - head - nvec * kVE;
@@ -137,22 +179,27 @@ __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n,
         blk = fmaf(x, x, blk);
     }
 
-    const uint4 *v = reinterpret_cast<const uint4 *>(seg + head * kEB);
+    const Vec *v = reinterpret_cast<const Vec *>(seg + head * kEB);
     double acc = 0.0;
     int64_t i = lane;
     int cnt = 0;
     for (; i + (kUnroll - 1) * 32 < nvec; i += kUnroll * 32) {
-        uint4 r[kUnroll];
+        Vec r[kUnroll];
 #pragma unroll
         for (int j = 0; j < kUnroll; ++j)
-            r[j] = ld_stream16(v + i + j * 32);
+            r[j] = ld_stream(v + i + j * 32);
         float a[kUnroll];
 #pragma unroll
         for (int j = 0; j < kUnroll; ++j) {
             a[j] = vec_sumsq<DT>(r[j]);
-            bits |= (r[j].x | r[j].y) | (r[j].z | r[j].w);
+            bits |= vec_or(r[j]);
         }
-        blk += ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
+#pragma unroll
+        for (int w = kUnroll / 2; w > 0; w >>= 1)     // pairwise tree
+#pragma unroll
+            for (int j = 0; j < w; ++j)
+                a[j] += a[j + w];
+        blk += a[0];
         if (++cnt == kFlush) {
             acc += static_cast<double>(blk);
             blk = 0.f;
@@ -161,15 +208,15 @@ __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n,
     }
     // Fewer than kUnroll vectors left for this lane: one predicated batch.
     {
-        uint4 r[kUnroll - 1];
+        Vec r[kUnroll - 1];
 #pragma unroll
         for (int j = 0; j < kUnroll - 1; ++j)
-            r[j] = (i + j * 32 < nvec) ? ld_stream16(v + i + j * 32) : make_uint4(0u, 0u, 0u, 0u);
+            r[j] = (i + j * 32 < nvec) ? ld_stream(v + i + j * 32) : zero_vec();
         float a = 0.f;
 #pragma unroll
         for (int j = 0; j < kUnroll - 1; ++j) {
             a += vec_sumsq<DT>(r[j]);
-            bits |= (r[j].x | r[j].y) | (r[j].z | r[j].w);
+            bits |= vec_or(r[j]);
         }
         blk += a;
     }
@@ -580,8 +627,8 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
 // sum of squares written to out_sumsq (the first half of a sharded step).
 // kStepFinish: no gradient read; phases 2-3 on the sums in in_sumsq (the
 // second half, after the caller has reduced the shards' sums).
-template <int DT, int MODE>
-__global__ void __launch_bounds__(kThreads, kMinCtasPerSm)
+template <int DT, int MODE, int V>
+__global__ void __launch_bounds__(kThreads, Shape<V>::kMinCtas)
 gnmr_step_kernel(const __grid_constant__ StepParams p)
 {
     __shared__ uint32_t s_hist[256];
@@ -647,7 +694,7 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
             const int64_t n = stop > pos ? stop - pos : 0;
             const char *seg = arena + (p.offset[g] + pos) * kEB;
             bool suspect;
-            double s = warp_segment_sumsq<DT>(seg, n, lane, suspect);
+            double s = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg, n, lane, suspect);
             if (suspect)
                 s = warp_segment_sumsq_f64<DT>(seg, n, lane);
             if (b != cur) {
@@ -681,34 +728,47 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     }
 }
 
-template <int MODE>
+template <int MODE, int V>
 cudaError_t launch_mode(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream)
 {
     if (dtype == 1)
-        gnmr_step_kernel<1, MODE><<<num_ctas, kThreads, 0, stream>>>(p);
+        gnmr_step_kernel<1, MODE, V><<<num_ctas, kThreads, 0, stream>>>(p);
     else
-        gnmr_step_kernel<0, MODE><<<num_ctas, kThreads, 0, stream>>>(p);
+        gnmr_step_kernel<0, MODE, V><<<num_ctas, kThreads, 0, stream>>>(p);
     return cudaGetLastError();
+}
+
+template <int V>
+cudaError_t launch_variant(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream, int mode)
+{
+    if (mode == kStepPartials)
+        return launch_mode<kStepPartials, V>(p, dtype, num_ctas, stream);
+    return launch_mode<kStepFull, V>(p, dtype, num_ctas, stream);
 }
 
 }  // namespace
 
-cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream, int mode)
+cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream, int mode,
+                        int variant)
 {
-    if (mode == kStepPartials)
-        return launch_mode<kStepPartials>(p, dtype, num_ctas, stream);
-    if (mode == kStepFinish)
-        return launch_mode<kStepFinish>(p, 0, num_ctas, stream);
-    return launch_mode<kStepFull>(p, dtype, num_ctas, stream);
+    if (mode == kStepFinish)                      // no gradient read: one shape is enough
+        return launch_mode<kStepFinish, kVariantSmall>(p, 0, num_ctas, stream);
+    if (variant == kVariantBulk)
+        return launch_variant<kVariantBulk>(p, dtype, num_ctas, stream, mode);
+    return launch_variant<kVariantSmall>(p, dtype, num_ctas, stream, mode);
 }
 
-cudaError_t step_occupancy(int dtype, int *ctas_per_sm)
+cudaError_t step_occupancy(int dtype, int variant, int *ctas_per_sm)
 {
-    if (dtype == 1)
-        return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<1, kStepFull>,
-                                                             kThreads, 0);
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<0, kStepFull>,
-                                                         kThreads, 0);
+    if (variant == kVariantBulk)
+        return dtype == 1 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                                ctas_per_sm, gnmr_step_kernel<1, kStepFull, kVariantBulk>, kThreads, 0)
+                          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                                ctas_per_sm, gnmr_step_kernel<0, kStepFull, kVariantBulk>, kThreads, 0);
+    return dtype == 1 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                            ctas_per_sm, gnmr_step_kernel<1, kStepFull, kVariantSmall>, kThreads, 0)
+                      : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+                            ctas_per_sm, gnmr_step_kernel<0, kStepFull, kVariantSmall>, kThreads, 0);
 }
 
 }  // namespace gnmr
