@@ -417,7 +417,7 @@ def run_gnmr(args):
                        "parallelism": "replicas" if world > 1 else "single GPU",
                        "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
                                f"{info['num_warps']} warp runs, "
-                               f"{'large-unit' if info['variant'] else 'small-unit'} loop shape"},
+                               f"{'large-unit' if info['loop_shape'] == 2 else 'small-unit'} loop shape"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
                          "traffic": traffic if w.name == "llama2-13b" and args.shrink == 1 else None,

@@ -87,7 +87,26 @@ typedef struct gnmr_config {
     /* Extra saved-activation cost c_b of recovering unit b (Eq.
      * generic-memory-bound), host [num_units], copied; NULL = no Delta M_t. */
     const double *unit_cost;
+    /* Shape of the kernel's streaming loop (gnmr_loop_shape).  The shapes
+     * split the arena into different warp runs, so norms agree within
+     * rounding, not bitwise; each shape is bitwise reproducible run to run.
+     * Default GNMR_LOOP_AUTO. */
+    int32_t loop_shape;
 } gnmr_config;
+
+/* Streaming-loop shapes of the step kernel.
+ *   GNMR_LOOP_AUTO: GNMR_LOOP_LARGE_UNITS when the mean unit holds at least
+ *     1 MiB of gradient, else GNMR_LOOP_SMALL_UNITS.
+ *   GNMR_LOOP_SMALL_UNITS: fewer loads in flight per warp, more resident
+ *     warps per SM (suits many small units, whose per-unit work overlaps the
+ *     stream of other warps).
+ *   GNMR_LOOP_LARGE_UNITS: twice the loads in flight per warp, half the
+ *     resident warps (suits long streams). */
+typedef enum gnmr_loop_shape {
+    GNMR_LOOP_AUTO = 0,
+    GNMR_LOOP_SMALL_UNITS = 1,
+    GNMR_LOOP_LARGE_UNITS = 2
+} gnmr_loop_shape;
 
 /* Recovery policies.
  *   GNMR_POLICY_ACTIVE_CAP (default): Algorithm 2, |A_t| <= maxO.
@@ -134,7 +153,7 @@ typedef struct gnmr_info {
     int64_t device_bytes;      /* library-owned device memory */
     int64_t arena_elems_min;   /* max over units of offset + length */
     int64_t steps;             /* gnmr_step calls enqueued so far */
-    int32_t variant;           /* streaming-loop shape: 0 many-small-units, 1 large units */
+    int32_t loop_shape;        /* gnmr_loop_shape in use (never GNMR_LOOP_AUTO) */
     int32_t reserved;
 } gnmr_info;
 

@@ -24,6 +24,7 @@ GNMR_DTYPE_BF16 = 1
 GNMR_FQ_NONE, GNMR_FQ_E2M1, GNMR_FQ_E3M2, GNMR_FQ_E4M3, GNMR_FQ_E5M2 = 0, 1, 2, 3, 4
 
 GNMR_POLICY_ACTIVE_CAP, GNMR_POLICY_ADMISSION_CAP, GNMR_POLICY_STATIC_TOP = 0, 1, 2
+GNMR_LOOP_AUTO, GNMR_LOOP_SMALL_UNITS, GNMR_LOOP_LARGE_UNITS = 0, 1, 2
 
 _P = ctypes.c_void_p
 
@@ -52,6 +53,7 @@ class gnmr_config(ctypes.Structure):
         ("static_warmup_steps", ctypes.c_int64),
         ("static_fraction", ctypes.c_double),
         ("unit_cost", _P),
+        ("loop_shape", ctypes.c_int32),
     ]
 
 
@@ -79,7 +81,7 @@ class gnmr_info(ctypes.Structure):
         ("device_bytes", ctypes.c_int64),
         ("arena_elems_min", ctypes.c_int64),
         ("steps", ctypes.c_int64),
-        ("variant", ctypes.c_int32),
+        ("loop_shape", ctypes.c_int32),
         ("reserved", ctypes.c_int32),
     ]
 

@@ -195,6 +195,8 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         c.static_warmup_steps < 0 || !(c.static_fraction >= 0.0 && c.static_fraction <= 1.0))
         return fail_create(GNMR_ERR_INVALID_ARG,
                            "policy, forced_recovery_steps, static_warmup_steps or static_fraction out of range");
+    if (c.loop_shape < GNMR_LOOP_AUTO || c.loop_shape > GNMR_LOOP_LARGE_UNITS)
+        return fail_create(GNMR_ERR_INVALID_ARG, "loop_shape out of range");
     if (c.unit_cost)
         for (int32_t b = 0; b < c.num_units; ++b)
             if (!std::isfinite(c.unit_cost[b]))
@@ -232,8 +234,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
     int64_t grad_bytes = 0;
     for (int64_t g = 0; g < S_in; ++g)
         grad_bytes += c.lengths[g] * eb;
-    const int variant = grad_bytes / c.num_units >= gnmr::kBulkUnitBytes ? gnmr::kVariantBulk
-                                                                         : gnmr::kVariantSmall;
+    const bool large = c.loop_shape == GNMR_LOOP_AUTO ? grad_bytes / c.num_units >= gnmr::kBulkUnitBytes
+                                                      : c.loop_shape == GNMR_LOOP_LARGE_UNITS;
+    const int variant = large ? gnmr::kVariantBulk : gnmr::kVariantSmall;
     int sms = 0, per_sm = 0;
     cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
     if (e == cudaSuccess)
@@ -646,7 +649,7 @@ gnmr_status gnmr_get_info(const gnmr_handle *h, gnmr_info *info)
     info->device_bytes = h->device_bytes;
     info->arena_elems_min = h->max_end;
     info->steps = h->steps;
-    info->variant = h->variant;
+    info->loop_shape = h->variant == gnmr::kVariantBulk ? GNMR_LOOP_LARGE_UNITS : GNMR_LOOP_SMALL_UNITS;
     info->reserved = 0;
     return GNMR_OK;
 }

@@ -2,6 +2,7 @@
 // and the device code (gnmr_kernels.cu).  Not part of the public ABI.
 #pragma once
 
+#include <cstddef>
 #include <cstdint>
 #include <vector>
 
@@ -38,6 +39,9 @@ struct UnitState {
     int32_t active;   // 1 if b was on the recovery path at the previous step
     double gsum;      // GNMR summed over the static policy's warm-up
 };
+// lock and active are written together as one 8-byte store
+static_assert(offsetof(UnitState, lock) % 8 == 0 && offsetof(UnitState, active) == offsetof(UnitState, lock) + 4,
+              "UnitState lock/active pair");
 
 // Candidate-pool entry written by the unit epilogue, read by the selection
 // (one 16-byte load).

@@ -249,6 +249,18 @@ __device__ __forceinline__ double pick_threshold(double override_value, int64_t 
     return t <= warmup ? init_value : main_value;
 }
 
+// Order-preserving keys: R >= 0 (never NaN), so its IEEE bits order like its
+// value; the low word ranks lower unit indices higher.
+__device__ __forceinline__ uint64_t risk_key(double r)
+{
+    const uint64_t bits = static_cast<uint64_t>(__double_as_longlong(r));
+    return (bits << 1) == 0 ? 0ull : bits;           // -0 and +0 share the key 0 (integer test)
+}
+__device__ __forceinline__ uint32_t index_key(int32_t b, int32_t num_units)
+{
+    return static_cast<uint32_t>(num_units - 1 - b);
+}
+
 // Unit epilogue for up to 32 units at once, one per lane (lanes with
 // `active` false only take part in the collective append): Algorithm 1, the
 // combined risk of Sec. 3.3, the statistics outputs and the candidate test of
@@ -333,6 +345,10 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
             if (t == p.static_warmup + 1 && rec) {
                 cand = true;                          // ranked once by the warm-up's GNMR sum
                 r = s.gsum;
+                // outcome if not kept (the last CTA rewrites the kept units)
+                p.mask[b] = 0;
+                p.state[b].active = 0;
+                if (p.out_lock) p.out_lock[b] = s.lock;
             } else {
                 p.mask[b] = (rec && t > p.static_warmup + 1 && s.active) ? 1 : 0;
                 if (t == p.static_warmup + 1)
@@ -341,12 +357,14 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
             }
         } else {
             cand = rec && (r > 1.0 || s.lock > 0);
-            if (!cand) {
-                // Not a candidate: Lock_b is already 0 and b stays on the low-cost path.
-                p.mask[b] = 0;
-                p.state[b].active = 0;
-                if (p.out_lock) p.out_lock[b] = 0;
-            }
+            // The outcome of a unit outside A_t (Algorithm 2: Lock_b = 0, low-cost
+            // path), written here for every unit; the last CTA rewrites only the
+            // selected ones.  A non-candidate's Lock_b is already 0.
+            p.mask[b] = 0;
+            p.state[b].active = 0;
+            if (cand)
+                p.state[b].lock = 0;
+            if (p.out_lock) p.out_lock[b] = 0;
         }
         cand_lock = static_cast<uint32_t>(s.lock) | (s.active ? kCandActive : 0u);
     }
@@ -395,17 +413,6 @@ __device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, in
     return true;
 }
 
-// Order-preserving keys: R >= 0 (never NaN), so its IEEE bits order like its
-// value; the low word ranks lower unit indices higher.
-__device__ __forceinline__ uint64_t risk_key(double r)
-{
-    return r == 0.0 ? 0ull : static_cast<uint64_t>(__double_as_longlong(r));
-}
-__device__ __forceinline__ uint32_t index_key(int32_t b, int32_t num_units)
-{
-    return static_cast<uint32_t>(num_units - 1 - b);
-}
-
 __device__ __forceinline__ void load_candidate(const Candidate *c, double &r, int32_t &b, uint32_t &lock)
 {
     const double2 v = __ldcg(reinterpret_cast<const double2 *>(c));
@@ -414,6 +421,47 @@ __device__ __forceinline__ void load_candidate(const Candidate *c, double &r, in
     b = static_cast<int32_t>(w & 0xffffffffu);
     lock = static_cast<uint32_t>(w >> 32);
 }
+
+// Bucket of the r-th largest digit in hist[256] (r >= 1): misc[1] = the
+// bucket, misc[2] = r minus the count above it, misc[3] = its count.  Warp 0
+// scans; the caller synchronises before and after.
+__device__ __forceinline__ void find_bucket(const uint32_t *hist, uint32_t r, uint32_t *misc)
+{
+    if (threadIdx.x >= 32)
+        return;
+    const int l = threadIdx.x;                       // lane l owns buckets 255-8l down to 248-8l
+    const uint4 *v = reinterpret_cast<const uint4 *>(hist + 248 - 8 * l);
+    const uint4 a = v[0], b = v[1];                  // buckets 248-8l .. 255-8l, ascending
+    const uint32_t c8[8] = {b.w, b.z, b.y, b.x, a.w, a.z, a.y, a.x};   // descending
+    uint32_t sum = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+        sum += c8[j];
+    uint32_t incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t v = __shfl_up_sync(kFull, incl, o);
+        if (l >= o)
+            incl += v;
+    }
+    const uint32_t excl = incl - sum;
+    if (excl < r && r <= incl) {                     // exactly one lane
+        uint32_t above = excl;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (above + c8[j] >= r) {
+                misc[1] = static_cast<uint32_t>(255 - 8 * l - j);
+                misc[2] = r - above;
+                misc[3] = c8[j];
+                break;
+            }
+            above += c8[j];
+        }
+    }
+}
+
+// Candidate loads a thread keeps in flight in each selection pass.
+constexpr int kSelectIlp = 6;
 
 // K-th largest 96-bit key (risk_key : index_key) among the m candidates (or
 // among those not active at t-1 when only_new), 1 <= K < that count, by
@@ -434,18 +482,18 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, bool o
         for (int i = threadIdx.x; i < 256; i += blockDim.x)
             hist[i] = 0;
         __syncthreads();
-        for (uint32_t i0 = threadIdx.x; i0 < m; i0 += 4 * blockDim.x) {
-            double rr[4];
-            int32_t bb[4];
-            uint32_t ll[4];
+        for (uint32_t i0 = threadIdx.x; i0 < m; i0 += kSelectIlp * blockDim.x) {
+            double rr[kSelectIlp];
+            int32_t bb[kSelectIlp];
+            uint32_t ll[kSelectIlp];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {           // four loads in flight per thread
+            for (int j = 0; j < kSelectIlp; ++j) {  // loads in flight per thread
                 const uint32_t i = i0 + j * blockDim.x;
                 if (i < m)
                     load_candidate(p.cand + i, rr[j], bb[j], ll[j]);
             }
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
+            for (int j = 0; j < kSelectIlp; ++j) {
                 if (i0 + j * blockDim.x >= m)
                     break;
                 if (only_new && (ll[j] & kCandActive))
@@ -460,36 +508,7 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, bool o
             }
         }
         __syncthreads();
-        if (threadIdx.x < 32) {
-            const int l = threadIdx.x;               // lane l owns buckets 255-8l down to 248-8l
-            uint32_t c8[8], sum = 0;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                c8[j] = hist[255 - 8 * l - j];
-                sum += c8[j];
-            }
-            uint32_t incl = sum;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const uint32_t v = __shfl_up_sync(kFull, incl, o);
-                if (l >= o)
-                    incl += v;
-            }
-            const uint32_t excl = incl - sum;
-            if (excl < r && r <= incl) {             // exactly one lane
-                uint32_t above = excl;
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    if (above + c8[j] >= r) {
-                        misc[1] = static_cast<uint32_t>(255 - 8 * l - j);
-                        misc[2] = r - above;
-                        misc[3] = c8[j];
-                        break;
-                    }
-                    above += c8[j];
-                }
-            }
-        }
+        find_bucket(hist, r, misc);
         __syncthreads();
         const uint32_t bucket = misc[1];
         const uint32_t in_bucket = misc[3];
@@ -542,9 +561,107 @@ __device__ void delta_mem(const StepParams &p, double *red)
         *p.out_delta_mem = red[0];
 }
 
+// Algorithm 2's outcome for a unit in A_t (the epilogue has already written
+// the outcome for every unit outside it).
+__device__ __forceinline__ void commit_selected(const StepParams &p, bool stat, int32_t b, double r, uint32_t lk)
+{
+    p.mask[b] = 1;
+    if (stat) {
+        p.state[b].active = 1;                       // the static policy keeps no locks
+    } else {
+        const int32_t prev = static_cast<int32_t>(lk & ~kCandActive);
+        const int32_t next = r > 1.0 ? p.lock_len : (prev - 1 > 0 ? prev - 1 : 0);
+        *reinterpret_cast<int2 *>(&p.state[b].lock) = make_int2(next, 1);   // lock, active
+        if (p.out_lock) p.out_lock[b] = next;
+    }
+}
+
+// The selecting CTA's copy of the candidates' risk keys: candidate i's
+// risk_key in keys[i] and whether it belongs to the capped pool in bit i of
+// pool_bits (the candidates outside it -- retained under the admission cap --
+// are selected without ranking).  One read of the candidate list fills it;
+// the radix passes then run on shared memory.
+constexpr uint32_t kKeyCache = 7168;
+constexpr size_t kKeyCacheBytes = sizeof(uint64_t) * kKeyCache + sizeof(uint32_t) * (kKeyCache / 32);
+
+__device__ __forceinline__ bool in_pool(const uint32_t *pool_bits, uint32_t i)
+{
+    return (pool_bits[i >> 5] >> (i & 31u)) & 1u;
+}
+
+// K-th largest (risk_key : index_key) among the pool's m <= kKeyCache cached
+// keys, 1 <= K < pool size: MSD radix select with 8-bit digits over the
+// cached 64-bit keys, then, only if whole keys tie at the cut, over the unit
+// indices (read from the candidate list).  Exactly K pool keys compare >= the
+// returned threshold.  All threads of the CTA call this.
+__device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K, const uint64_t *keys,
+                                    const uint32_t *pool_bits, uint32_t *hist, uint32_t *misc,
+                                    uint64_t &thr_hi, uint32_t &thr_lo)
+{
+    const int lo_bits = p.num_units > 1 ? 32 - __clz(static_cast<uint32_t>(p.num_units - 1)) : 0;
+    const int lo_digits = (lo_bits + 7) / 8;
+    const uint32_t lane = threadIdx.x & 31u;
+    uint64_t pre_hi = 0, msk_hi = 0;
+    uint32_t pre_lo = 0, msk_lo = 0;
+    uint32_t r = K;
+    for (int dgt = 0; dgt < 8 + lo_digits; ++dgt) {
+        const bool in_hi = dgt < 8;
+        const int shift = in_hi ? 56 - 8 * dgt : 8 * (lo_digits - 1 - (dgt - 8));
+        for (int i = threadIdx.x; i < 256; i += blockDim.x)
+            hist[i] = 0;
+        __syncthreads();
+        // four keys per thread per iteration (independent chains)
+        for (uint32_t w0 = threadIdx.x & ~31u; w0 < m; w0 += 4 * blockDim.x) {
+            bool take[4];
+            uint32_t dig[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint32_t i = w0 + j * blockDim.x + lane;
+                take[j] = i < m && in_pool(pool_bits, i);
+                dig[j] = 0;
+                if (take[j]) {
+                    const uint64_t hi = keys[i];
+                    take[j] = (hi & msk_hi) == pre_hi;
+                    if (in_hi) {
+                        dig[j] = static_cast<uint32_t>(hi >> shift) & 0xffu;
+                    } else if (take[j]) {           // whole keys tie: rank by unit index
+                        const uint32_t lo = index_key(__ldcg(&p.cand[i].unit), p.num_units);
+                        take[j] = (lo & msk_lo) == pre_lo;
+                        dig[j] = (lo >> shift) & 0xffu;
+                    }
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (take[j])
+                    atomicAdd(&hist[dig[j]], 1u);
+        }
+        __syncthreads();
+        find_bucket(hist, r, misc);
+        __syncthreads();
+        const uint32_t bucket = misc[1];
+        const uint32_t in_bucket = misc[3];
+        r = misc[2];
+        if (in_hi) {
+            pre_hi |= static_cast<uint64_t>(bucket) << shift;
+            msk_hi |= 0xffull << shift;
+        } else {
+            pre_lo |= bucket << shift;
+            msk_lo |= 0xffu << shift;
+        }
+        __syncthreads();
+        if (in_bucket == r)                          // every key with this prefix is in
+            break;
+    }
+    thr_hi = pre_hi;
+    thr_lo = pre_lo;
+}
+
 // Last CTA: Top_maxO (or the policy's choice), Algorithm 2's lock
-// bookkeeping, mask, counts, Delta M_t, reset.
-__device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist, uint32_t *misc, double *red)
+// bookkeeping, mask, counts, Delta M_t, reset.  The unit epilogues have
+// already written the outcome of every unit outside A_t; this writes A_t.
+__device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist, uint32_t *misc, double *red,
+                                  unsigned char *key_cache)
 {
     uint32_t m = __ldcg(&p.ctl->n_cand);
     m = m < static_cast<uint32_t>(p.num_units) ? m : static_cast<uint32_t>(p.num_units);
@@ -572,37 +689,78 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
         const uint32_t cap = stat ? static_cast<uint32_t>(p.static_keep) : static_cast<uint32_t>(p.max_o);
         const uint32_t K = pool < cap ? pool : cap;
         const bool take_all = pool <= cap;
-        uint64_t thr_hi = 0;
-        uint32_t thr_lo = 0;
-        if (!take_all && K > 0)
-            radix_select(p, m, K, admission, hist, misc, thr_hi, thr_lo);
-        for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
-            double r;
-            int32_t b;
-            uint32_t lk;
-            load_candidate(p.cand + i, r, b, lk);
-            const bool was_active = (lk & kCandActive) != 0;
-            const int32_t prev = static_cast<int32_t>(lk & ~kCandActive);
-            bool sel;
-            if (admission && was_active) {
-                sel = true;                              // retained without counting against the cap
-            } else if (take_all) {
-                sel = true;
-            } else if (K == 0) {
-                sel = false;
-            } else {
-                const uint64_t hi = risk_key(r);
-                sel = hi > thr_hi || (hi == thr_hi && index_key(b, p.num_units) >= thr_lo);
+        if (take_all || K == 0) {
+            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+                double r;
+                int32_t b;
+                uint32_t lk;
+                load_candidate(p.cand + i, r, b, lk);
+                if (take_all || (admission && (lk & kCandActive)))
+                    commit_selected(p, stat, b, r, lk);
             }
-            int32_t next;
-            if (stat)
-                next = prev;                             // the static policy keeps no locks
-            else
-                next = !sel ? 0 : (r > 1.0 ? p.lock_len : (prev - 1 > 0 ? prev - 1 : 0));
-            p.state[b].lock = next;
-            p.state[b].active = sel ? 1 : 0;
-            p.mask[b] = sel ? 1 : 0;
-            if (p.out_lock) p.out_lock[b] = next;
+        } else if (m <= kKeyCache) {
+            uint64_t *keys = reinterpret_cast<uint64_t *>(key_cache);
+            uint32_t *pool_bits = reinterpret_cast<uint32_t *>(key_cache + sizeof(uint64_t) * kKeyCache);
+            const uint32_t lane = threadIdx.x & 31u;
+            // one read of the candidate list (loads in flight per thread)
+            for (uint32_t w0 = (threadIdx.x & ~31u); w0 < m; w0 += kSelectIlp * blockDim.x) {
+                double rr[kSelectIlp];
+                uint32_t ll[kSelectIlp];
+#pragma unroll
+                for (int j = 0; j < kSelectIlp; ++j) {
+                    const uint32_t i = w0 + j * blockDim.x + lane;
+                    int32_t b;
+                    if (i < m)
+                        load_candidate(p.cand + i, rr[j], b, ll[j]);
+                }
+#pragma unroll
+                for (int j = 0; j < kSelectIlp; ++j) {
+                    const uint32_t i = w0 + j * blockDim.x + lane;
+                    const bool member = i < m && !(admission && (ll[j] & kCandActive));
+                    const unsigned word = __ballot_sync(kFull, member);
+                    if (i < m)
+                        keys[i] = risk_key(rr[j]);
+                    if (lane == 0 && w0 + j * blockDim.x < m)
+                        pool_bits[(w0 + j * blockDim.x) >> 5] = word;
+                }
+            }
+            __syncthreads();
+            uint64_t thr_hi = 0;
+            uint32_t thr_lo = 0;
+            radix_select_cached(p, m, K, keys, pool_bits, hist, misc, thr_hi, thr_lo);
+            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+                bool sel;
+                if (!in_pool(pool_bits, i)) {
+                    sel = true;                              // retained outside the cap
+                } else {
+                    const uint64_t key = keys[i];
+                    sel = key > thr_hi ||
+                          (key == thr_hi && index_key(__ldcg(&p.cand[i].unit), p.num_units) >= thr_lo);
+                }
+                if (sel) {
+                    double r;
+                    int32_t b;
+                    uint32_t lk;
+                    load_candidate(p.cand + i, r, b, lk);
+                    commit_selected(p, stat, b, r, lk);
+                }
+            }
+        } else {
+            // more candidates than the shared-memory cache: radix passes over
+            // the candidate list in global memory
+            uint64_t thr_hi = 0;
+            uint32_t thr_lo = 0;
+            radix_select(p, m, K, admission, hist, misc, thr_hi, thr_lo);
+            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+                double r;
+                int32_t b;
+                uint32_t lk;
+                load_candidate(p.cand + i, r, b, lk);
+                const uint64_t key = risk_key(r);
+                if ((admission && (lk & kCandActive)) || key > thr_hi ||
+                    (key == thr_hi && index_key(b, p.num_units) >= thr_lo))
+                    commit_selected(p, stat, b, r, lk);
+            }
         }
         n_sel = K + retained;
     }
@@ -631,9 +789,10 @@ template <int DT, int MODE, int V>
 __global__ void __launch_bounds__(kThreads, Shape<V>::kMinCtas)
 gnmr_step_kernel(const __grid_constant__ StepParams p)
 {
-    __shared__ uint32_t s_hist[256];
+    __shared__ __align__(16) uint32_t s_hist[256];
     __shared__ uint32_t s_misc[8];
     __shared__ double s_red[kThreads];
+    extern __shared__ __align__(16) unsigned char s_keys[];   // kKeyCacheBytes unless MODE == kStepPartials
     constexpr int kEB = Elem<DT>::kBytes;
     const int lane = threadIdx.x & 31;
     const int warp = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
@@ -724,17 +883,18 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     __syncthreads();
     if (s_misc[0]) {
         __threadfence();
-        select_and_commit(p, __ldcg(&p.ctl->steps) + 1, s_hist, s_misc, s_red);
+        select_and_commit(p, __ldcg(&p.ctl->steps) + 1, s_hist, s_misc, s_red, s_keys);
     }
 }
 
 template <int MODE, int V>
 cudaError_t launch_mode(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream)
 {
+    constexpr size_t smem = MODE == kStepPartials ? 0 : kKeyCacheBytes;
     if (dtype == 1)
-        gnmr_step_kernel<1, MODE, V><<<num_ctas, kThreads, 0, stream>>>(p);
+        gnmr_step_kernel<1, MODE, V><<<num_ctas, kThreads, smem, stream>>>(p);
     else
-        gnmr_step_kernel<0, MODE, V><<<num_ctas, kThreads, 0, stream>>>(p);
+        gnmr_step_kernel<0, MODE, V><<<num_ctas, kThreads, smem, stream>>>(p);
     return cudaGetLastError();
 }
 
@@ -758,17 +918,35 @@ cudaError_t launch_step(const StepParams &p, int dtype, int num_ctas, cudaStream
     return launch_variant<kVariantSmall>(p, dtype, num_ctas, stream, mode);
 }
 
+namespace {
+
+// The key cache is dynamic shared memory above the 48 KiB default, an opt-in
+// that is a per-device function attribute: set for every instance a handle
+// launches, on the current device.
+template <int DT, int V>
+cudaError_t prepare_variant(int *ctas_per_sm)
+{
+    const int bytes = static_cast<int>(kKeyCacheBytes);
+    cudaError_t e = cudaFuncSetAttribute(gnmr_step_kernel<DT, kStepFull, V>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(gnmr_step_kernel<0, kStepFinish, kVariantSmall>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, gnmr_step_kernel<DT, kStepFull, V>,
+                                                          kThreads, kKeyCacheBytes);
+    return e;
+}
+
+}  // namespace
+
 cudaError_t step_occupancy(int dtype, int variant, int *ctas_per_sm)
 {
     if (variant == kVariantBulk)
-        return dtype == 1 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-                                ctas_per_sm, gnmr_step_kernel<1, kStepFull, kVariantBulk>, kThreads, 0)
-                          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-                                ctas_per_sm, gnmr_step_kernel<0, kStepFull, kVariantBulk>, kThreads, 0);
-    return dtype == 1 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-                            ctas_per_sm, gnmr_step_kernel<1, kStepFull, kVariantSmall>, kThreads, 0)
-                      : cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-                            ctas_per_sm, gnmr_step_kernel<0, kStepFull, kVariantSmall>, kThreads, 0);
+        return dtype == 1 ? prepare_variant<1, kVariantBulk>(ctas_per_sm)
+                          : prepare_variant<0, kVariantBulk>(ctas_per_sm);
+    return dtype == 1 ? prepare_variant<1, kVariantSmall>(ctas_per_sm)
+                      : prepare_variant<0, kVariantSmall>(ctas_per_sm);
 }
 
 }  // namespace gnmr

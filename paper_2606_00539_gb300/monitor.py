@@ -10,6 +10,8 @@ from . import _native as N
 
 _DTYPES = {"f32": N.GNMR_DTYPE_F32, "float32": N.GNMR_DTYPE_F32,
            "bf16": N.GNMR_DTYPE_BF16, "bfloat16": N.GNMR_DTYPE_BF16}
+_LOOP_SHAPES = {"auto": N.GNMR_LOOP_AUTO, "small": N.GNMR_LOOP_SMALL_UNITS,
+                "large": N.GNMR_LOOP_LARGE_UNITS}
 
 
 def _torch():
@@ -29,13 +31,14 @@ class Monitor:
     t <= warmup_steps (two-stage schedule).  A scalar means both stages.
     policy, forced_recovery_steps, static_warmup_steps, static_fraction: the
     recovery policy variants of include/gnmr.h; unit_cost: per-unit c_b for
-    the Delta M_t statistic.
+    the Delta M_t statistic.  loop_shape: "auto", "small" or "large", the
+    kernel's streaming-loop shape (norms agree within rounding across shapes).
     """
 
     def __init__(self, offsets, lengths, *, dtype="bf16", recoverable=None, window=8, max_o=4,
                  lock_len=1, alpha=(1.5, 1.1), beta=(1.5, 1.5), warmup_steps=0, eps=1e-8,
                  device=0, segment_unit=None, num_units=None, policy=0, forced_recovery_steps=0,
-                 static_warmup_steps=0, static_fraction=0.25, unit_cost=None):
+                 static_warmup_steps=0, static_fraction=0.25, unit_cost=None, loop_shape="auto"):
         self._h = None
         off = np.ascontiguousarray(offsets, dtype=np.int64)
         ln = np.ascontiguousarray(lengths, dtype=np.int64)
@@ -83,6 +86,9 @@ class Monitor:
         cfg.forced_recovery_steps = int(forced_recovery_steps)
         cfg.static_warmup_steps = int(static_warmup_steps)
         cfg.static_fraction = float(static_fraction)
+        if loop_shape not in _LOOP_SHAPES:
+            raise ValueError(f"loop_shape must be one of {sorted(_LOOP_SHAPES)}")
+        cfg.loop_shape = _LOOP_SHAPES[loop_shape]
         cost = None
         if unit_cost is not None:
             cost = np.ascontiguousarray(unit_cost, dtype=np.float64)

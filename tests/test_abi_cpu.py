@@ -63,13 +63,13 @@ int main(void) {
   F(gnmr_config, warmup_steps) F(gnmr_config, eps) F(gnmr_config, device)
   F(gnmr_config, num_segments) F(gnmr_config, segment_unit) F(gnmr_config, policy)
   F(gnmr_config, forced_recovery_steps) F(gnmr_config, static_warmup_steps)
-  F(gnmr_config, static_fraction) F(gnmr_config, unit_cost)
+  F(gnmr_config, static_fraction) F(gnmr_config, unit_cost) F(gnmr_config, loop_shape)
   F(gnmr_stats, norm) F(gnmr_stats, gnmr) F(gnmr_stats, dgnmr) F(gnmr_stats, risk)
   F(gnmr_stats, lock) F(gnmr_stats, counts) F(gnmr_stats, delta_mem)
   F(gnmr_info, num_units) F(gnmr_info, dtype) F(gnmr_info, device) F(gnmr_info, num_ctas)
   F(gnmr_info, threads_per_cta) F(gnmr_info, num_warps) F(gnmr_info, num_partials)
   F(gnmr_info, device_bytes) F(gnmr_info, arena_elems_min) F(gnmr_info, steps)
-  F(gnmr_info, variant) F(gnmr_info, reserved)
+  F(gnmr_info, loop_shape) F(gnmr_info, reserved)
   return 0;
 }
 """
@@ -112,6 +112,7 @@ def _valid_cfg(off, ln):
     ("alpha_init", 0.0), ("alpha_main", float("inf")), ("beta_init", -1.0),
     ("beta_main", float("nan")), ("eps", -1e-3), ("warmup_steps", -5), ("policy", 3),
     ("forced_recovery_steps", -1), ("static_fraction", 1.5), ("static_warmup_steps", -2),
+    ("loop_shape", 3), ("loop_shape", -1),
 ])
 def test_create_rejects_bad_config_before_cuda(lib, field, value):
     off = np.array([0, 10], np.int64)
@@ -239,3 +240,9 @@ def test_partition_rejects_bad_input(lib):
         N.gnmr_plan_partition(np.array([5, -1], np.int64), N.GNMR_DTYPE_F32, 4)
     with pytest.raises(N.GnmrError):
         N.gnmr_plan_partition(np.array([5], np.int64), 9, 4)
+
+
+def test_monitor_rejects_unknown_loop_shape(lib):
+    from paper_2606_00539_gb300 import Monitor
+    with pytest.raises(ValueError, match="loop_shape"):
+        Monitor(np.array([0], np.int64), np.array([4], np.int64), loop_shape="medium")

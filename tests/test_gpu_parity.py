@@ -77,6 +77,44 @@ def test_block_level_units_parity(config, group, shrink, steps, cuda_device):
     _run_lockstep(w)
 
 
+def _large_shape_monitor(w, **over):
+    return _monitor(w, loop_shape="large", **over)
+
+
+@pytest.mark.parametrize("config,group,shrink,steps", [
+    ("tiny", "tensor", 1, 60),
+    ("llama2-13b", "tensor", 16, None),
+    ("aq-stress", "tensor", 1, 10),
+    ("moe", "expert", 16, 12),
+])
+def test_large_unit_loop_shape_parity(config, group, shrink, steps, cuda_device):
+    """The large-unit loop shape (twice the loads in flight per warp, half
+    the resident warps) forced on the small cases, which would otherwise run
+    the small-unit shape: same bar against the oracle."""
+    w = workloads.make(config, shrink=shrink, steps=steps, group=group)
+    tr = TD.LockstepTrace(w, "cuda:0", _large_shape_monitor)
+    try:
+        assert tr.mon.info()["loop_shape"] == N.GNMR_LOOP_LARGE_UNITS
+        for t in range(w.steps):
+            norms, res, got = tr.step(t)
+            TD.compare(norms, res, got, RTOL)
+    finally:
+        tr.close()
+
+
+def test_loop_shape_follows_the_mean_unit_size(cuda_device):
+    """GNMR_LOOP_AUTO takes the large-unit shape at >= 1 MiB per unit."""
+    for config, want in (("tiny", N.GNMR_LOOP_SMALL_UNITS), ("aq-stress", N.GNMR_LOOP_SMALL_UNITS),
+                         ("llama2-1.3b", N.GNMR_LOOP_LARGE_UNITS), ("llama2-13b", N.GNMR_LOOP_LARGE_UNITS),
+                         ("moe", N.GNMR_LOOP_LARGE_UNITS)):
+        w = workloads.make(config)
+        with _monitor(w) as mon:
+            assert mon.info()["loop_shape"] == want, config
+        for shape, code in (("small", N.GNMR_LOOP_SMALL_UNITS), ("large", N.GNMR_LOOP_LARGE_UNITS)):
+            with _monitor(w, loop_shape=shape) as mon:
+                assert mon.info()["loop_shape"] == code
+
+
 def test_segments_in_any_order_and_units_without_segments(cuda_device):
     import torch
     rng = np.random.default_rng(21)
@@ -203,8 +241,9 @@ def _parity_on_norms(off, ln, dev_arena, make_step, mon_kw, ctl_kw, steps, recov
         ctl.close()
 
 
+@pytest.mark.parametrize("shape", ["small", "large"])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_unaligned_overlapping_and_empty_units(dtype, cuda_device):
+def test_unaligned_overlapping_and_empty_units(dtype, shape, cuda_device):
     """Units at odd element offsets, overlapping units, gaps, zero-length and
     one-element units, and a unit spanning many warps."""
     import torch
@@ -228,7 +267,8 @@ def test_unaligned_overlapping_and_empty_units(dtype, cuda_device):
         dev.copy_(x.to(dev.dtype))
 
     _parity_on_norms(off, ln, dev, make_step,
-                     dict(dtype=dtype, window=2, max_o=3, lock_len=2, alpha=1.2, beta=1.2),
+                     dict(dtype=dtype, window=2, max_o=3, lock_len=2, alpha=1.2, beta=1.2,
+                          loop_shape=shape),
                      dict(window=2, max_o=3, lock_len=2, alpha=(1.2, 1.2), beta=(1.2, 1.2)), 6)
 
 
@@ -293,7 +333,8 @@ def test_budget_extremes_and_ties(max_o, lock_len, thr, cuda_device):
                      8, recoverable=rec)
 
 
-def test_tiny_and_huge_fp32_values_take_the_exact_path(cuda_device):
+@pytest.mark.parametrize("shape", ["small", "large"])
+def test_tiny_and_huge_fp32_values_take_the_exact_path(shape, cuda_device):
     """fp32 squares underflow below ~1e-19 and overflow above ~1.8e19; the
     kernel's fp64 fallback keeps the norm within rounding of the oracle."""
     import torch
@@ -305,7 +346,7 @@ def test_tiny_and_huge_fp32_values_take_the_exact_path(cuda_device):
     off = np.cumsum([0] + [len(p) for p in parts[:-1]]).astype(np.int64)
     ln = np.array([len(p) for p in parts], np.int64)
     dev = torch.from_numpy(host).to(cuda_device)
-    mon = Monitor(off, ln, dtype="f32", device=0)
+    mon = Monitor(off, ln, dtype="f32", device=0, loop_shape=shape)
     stats = mon.new_stats()
     try:
         mon.step(dev, stats=stats)
@@ -353,14 +394,15 @@ def test_threshold_override_and_schedule(cuda_device):
         tr.close()
 
 
-def test_deterministic_across_handles_and_runs(cuda_device):
+@pytest.mark.parametrize("shape", ["small", "large"])
+def test_deterministic_across_handles_and_runs(shape, cuda_device):
     import torch
     w = workloads.make("llama2-13b", shrink=32, steps=4)
     f = workloads.Filler(w, cuda_device)
     arena = f.new_arena()
     outs = []
     for _ in range(2):
-        mon = _monitor(w)
+        mon = _monitor(w, loop_shape=shape)
         stats = mon.new_stats()
         vals = []
         for t in range(w.steps):
