@@ -353,6 +353,7 @@ def run_gnmr(args):
     # end to end through the public API: host arena (pinned) -> device, the
     # step, the mask back to the host, every step inside the timed region
     e2e = None
+    e2e_in_place = None
     host = None
     if not args.no_e2e and args.e2e_steps > 0:
         try:
@@ -379,6 +380,27 @@ def run_gnmr(args):
                    "h2d_bytes_per_step": int(host.numel() * host.element_size()),
                    "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
                    "path": "pinned host arena -> device copy, gnmr_step, mask -> pinned host"}
+            # the same public call reading the pinned host arena in place: the
+            # kernel's loads cross the host link, no staging copy or device
+            # buffer for the gradients
+            for i in range(args.e2e_steps + 1):
+                if i == 1:
+                    torch.cuda.synchronize(dev)
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                with torch.cuda.stream(stream):
+                    mon.step(host, mask=mask, stream=stream)
+                    host_mask.copy_(mask, non_blocking=True)
+                stream.synchronize()
+            e1.record(stream)
+            stream.synchronize()
+            ip_ms = max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
+            e2e_in_place = {"value": round(world * gbytes / (ip_ms / 1e3), 3), "unit": "GB/s",
+                            "ms_per_step": round(ip_ms, 3),
+                            "h2d_bytes_per_step": int(host.numel() * host.element_size()),
+                            "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
+                            "path": "gnmr_step reading the pinned host arena in place, mask -> pinned host"}
         except RuntimeError as exc:
             e2e = {"value": None, "unit": "GB/s", "error": str(exc).splitlines()[0]}
             host = None
@@ -428,6 +450,7 @@ def run_gnmr(args):
                          "kernel_ms_min": round(min(per_ms), 4)},
             "cpu_baseline": cpu,
             "e2e": e2e,
+            "e2e_in_place": e2e_in_place,
             "gpu_launches": launches,
             "clocks": clocks,
         }

@@ -188,9 +188,14 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out);
  * A unit whose norm is NaN or Inf gets GNMR = Delta-GNMR = R = +Inf and its
  * A_b, Q_b and k_b are left as they were.
  * Arguments:
- *   d_arena      device, the flat gradient arena of the configured dtype,
- *                aligned to its element size; read only.  May be NULL only
- *                if every unit is empty.
+ *   d_arena      device-accessible, the flat gradient arena of the
+ *                configured dtype, aligned to its element size; read only.
+ *                Device memory, or pinned host memory (cudaHostAlloc, or
+ *                cudaHostRegister'ed; under unified addressing its host
+ *                address is its device address): a host arena is read in
+ *                place over the host link, with no staging copy and no
+ *                device memory for the gradients; results are bitwise the
+ *                same.  May be NULL only if every unit is empty.
  *   arena_elems  elements in d_arena; must be >= max(offset + length)
  *                (else GNMR_ERR_LAYOUT).
  *   stream       cudaStream_t as void*; NULL = legacy default stream.

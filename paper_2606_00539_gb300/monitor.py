@@ -179,13 +179,12 @@ class Monitor:
         """First half of a sharded step: per-unit sums of squares of this
         rank's local arena (fp64 tensor [U]); no controller state changes."""
         torch = _torch()
-        want = torch.bfloat16 if self.dtype == N.GNMR_DTYPE_BF16 else torch.float32
-        self._check_tensor(arena, "arena", want)
+        dev = self._check_arena(arena)
         if sumsq is None:
-            sumsq = torch.empty(self.num_units, dtype=torch.float64, device=arena.device)
+            sumsq = torch.empty(self.num_units, dtype=torch.float64, device=dev)
         self._check_tensor(sumsq, "sumsq", torch.float64, self.num_units)
         N.gnmr_step_partials(self._h, arena.data_ptr(), arena.numel(),
-                             self._stream_handle(stream, arena.device), sumsq.data_ptr())
+                             self._stream_handle(stream, dev), sumsq.data_ptr())
         return sumsq
 
     def finish(self, sumsq, mask=None, stats: dict | None = None, stream=None):
@@ -208,15 +207,31 @@ class Monitor:
         torch = _torch()
         N.gnmr_set_state(self._h, blob, self._stream_handle(stream, torch.device("cuda", self.device_index)))
 
-    def step(self, arena, mask=None, stats: dict | None = None, stream=None):
-        """Enqueues one GNMR step on `stream` (default: torch's current
-        stream) and returns the uint8 mask tensor (1 = recovery path)."""
+    def _check_arena(self, arena):
+        """The arena: a CUDA tensor on the handle's device, or a pinned CPU
+        tensor, which the kernel reads in place over the host link."""
         torch = _torch()
         want = torch.bfloat16 if self.dtype == N.GNMR_DTYPE_BF16 else torch.float32
-        self._check_tensor(arena, "arena", want)
+        if isinstance(arena, torch.Tensor) and not arena.is_cuda:
+            if not arena.is_pinned():
+                raise ValueError("a host arena must be pinned (pin_memory=True)")
+            if arena.dtype != want:
+                raise ValueError(f"arena must be {want}, got {arena.dtype}")
+            if not arena.is_contiguous():
+                raise ValueError("arena must be contiguous")
+        else:
+            self._check_tensor(arena, "arena", want)
+        return torch.device("cuda", self.device_index)
+
+    def step(self, arena, mask=None, stats: dict | None = None, stream=None):
+        """Enqueues one GNMR step on `stream` (default: torch's current
+        stream) and returns the uint8 mask tensor (1 = recovery path).
+        `arena` is a CUDA tensor or a pinned CPU tensor (read in place)."""
+        torch = _torch()
+        dev = self._check_arena(arena)
         if mask is None:
-            mask = torch.empty(self.num_units, dtype=torch.uint8, device=arena.device)
+            mask = torch.empty(self.num_units, dtype=torch.uint8, device=dev)
         self._check_tensor(mask, "mask", torch.uint8, self.num_units)
-        N.gnmr_step(self._h, arena.data_ptr(), arena.numel(), self._stream_handle(stream, arena.device),
+        N.gnmr_step(self._h, arena.data_ptr(), arena.numel(), self._stream_handle(stream, dev),
                     mask.data_ptr(), self._stats_struct(stats))
         return mask

@@ -394,6 +394,40 @@ def test_threshold_override_and_schedule(cuda_device):
         tr.close()
 
 
+@pytest.mark.parametrize("config,shrink", [("llama2-13b", 32), ("tiny", 1), ("moe", 32)])
+def test_pinned_host_arena_is_read_in_place(config, shrink, cuda_device):
+    """gnmr_step on a pinned host arena (read in place over the host link)
+    gives bitwise the outputs of the same arena in device memory, and so do
+    the partial sums; an unpinned host tensor is refused."""
+    import torch
+    w = workloads.make(config, shrink=shrink, steps=4)
+    f = workloads.Filler(w, cuda_device)
+    arena = f.new_arena()
+    host = torch.empty(arena.numel(), dtype=arena.dtype, pin_memory=True)
+    m_dev, m_host = _monitor(w), _monitor(w)
+    s_dev, s_host = m_dev.new_stats(), m_host.new_stats()
+
+    def bits(x):
+        return x.view(torch.int64) if x.dtype == torch.float64 else x
+
+    try:
+        for t in range(w.steps):
+            f.fill(arena, t)
+            host.copy_(arena)
+            a = m_dev.step(arena, stats=s_dev)
+            b = m_host.step(host, stats=s_host)
+            torch.cuda.synchronize()
+            assert torch.equal(a, b), f"mask, step {t + 1}"
+            for k in s_dev:
+                assert torch.equal(bits(s_dev[k]), bits(s_host[k])), f"{k}, step {t + 1}"
+        assert torch.equal(bits(m_dev.step_partials(arena)), bits(m_host.step_partials(host)))
+        with pytest.raises(ValueError, match="pinned"):
+            m_host.step(torch.zeros(8, dtype=arena.dtype))
+    finally:
+        m_dev.close()
+        m_host.close()
+
+
 @pytest.mark.parametrize("shape", ["small", "large"])
 def test_deterministic_across_handles_and_runs(shape, cuda_device):
     import torch
