@@ -54,12 +54,18 @@ def parse_args(argv=None):
     p.add_argument("--flush-l2", action="store_true",
                    help="write 512 MB before every timed step (outside its events)")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--graph", action="store_true",
+                   help="capture the K timed steps (K gnmr_step launches) in one CUDA graph and "
+                        "replay it: no host gaps between steps")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-units", type=int, default=0,
                    help="units in the CPU-oracle sample (0 = all: one full step)")
     p.add_argument("--ref-sample-units", type=int, default=42,
                    help="units per step of the reference arm (host-generated)")
-    return p.parse_args(argv)
+    args = p.parse_args(argv)
+    if args.graph and args.flush_l2:
+        p.error("--graph times back-to-back steps; it does not combine with --flush-l2")
+    return args
 
 
 # ---------------------------------------------------------------------------
@@ -310,6 +316,15 @@ def run_gnmr(args):
         mon.step(arenas[i % n_arenas], mask=mask, stats=stats, stream=stream)
     stream.synchronize()
 
+    graph = None
+    if args.graph:
+        # the captured steps run (and advance the controller) only when replayed
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for i in range(args.steps):
+                mon.step(arenas[(args.warmup + i) % n_arenas], mask=mask, stats=stats, stream=stream)
+        torch.cuda.synchronize(dev)
+
     sampler = ClockSampler(local_rank)
     time.sleep(0.3)                       # let nvidia-smi start sampling
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -320,15 +335,21 @@ def run_gnmr(args):
     torch.cuda.synchronize(dev)
     wall0 = time.time()
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if args.flush_l2 else None
-    t_start.record(stream)
-    for i in range(args.steps):
-        if flush is not None:
-            with torch.cuda.stream(stream):
-                flush.zero_()
-        ev[i][0].record(stream)
-        mon.step(arenas[(args.warmup + i) % n_arenas], mask=mask, stats=stats, stream=stream)
-        ev[i][1].record(stream)
-    t_end.record(stream)
+    if graph is not None:
+        t_start.record(stream)
+        with torch.cuda.stream(stream):
+            graph.replay()
+        t_end.record(stream)
+    else:
+        t_start.record(stream)
+        for i in range(args.steps):
+            if flush is not None:
+                with torch.cuda.stream(stream):
+                    flush.zero_()
+            ev[i][0].record(stream)
+            mon.step(arenas[(args.warmup + i) % n_arenas], mask=mask, stats=stats, stream=stream)
+            ev[i][1].record(stream)
+        t_end.record(stream)
     stream.synchronize()
     torch.cuda.synchronize(dev)
     wall1 = time.time()
@@ -336,7 +357,11 @@ def run_gnmr(args):
     sampler.stop()
     clocks = sampler.summary(wall0, wall1)
 
-    per_ms = [a.elapsed_time(b) for a, b in ev]
+    if graph is not None:
+        # back-to-back launches of one kernel: its mean duration is the region / K
+        per_ms = [t_start.elapsed_time(t_end) / args.steps] * args.steps
+    else:
+        per_ms = [a.elapsed_time(b) for a, b in ev]
     # with flushes in the region, the step time is the sum of the steps' own events
     total_ms = sum(per_ms) if flush is not None else t_start.elapsed_time(t_end)
     max_ms = max_over_ranks(total_ms, world, dev)
@@ -437,6 +462,8 @@ def run_gnmr(args):
                               else "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * 129e6
                               else "inputs fit in L2 (hot)"),
                        "parallelism": "replicas" if world > 1 else "single GPU",
+                       "launch": ("one CUDA graph of the timed steps, replayed" if args.graph
+                                  else "one gnmr_step call per step"),
                        "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
                                f"{info['num_warps']} warp runs, "
                                f"{'large-unit' if info['loop_shape'] == 2 else 'small-unit'} loop shape"},

@@ -27,7 +27,7 @@ constexpr int64_t kBulkUnitBytes = int64_t(1) << 20;
 // smaller than kMinRunBytes unless the whole problem is.
 constexpr int64_t kUnitCostBytes = 4096;
 constexpr int64_t kSplitBytes = 512;
-constexpr int64_t kMinRunBytes = 16384;
+constexpr int64_t kMinRunBytes = 4096;   // one 4 KiB load round per warp: small problems spread over more SMs
 
 // Persistent per-unit controller state (Algorithm 1 and 2), 40 bytes.
 struct UnitState {
