@@ -275,6 +275,12 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
     uint32_t cand_lock = 0;
     if (active) {
         const double n = sqrt(sumsq);
+        const int w = p.window;
+        double *Q = p.queue + static_cast<int64_t>(b) * w;
+        // the window's lines travel with the state load: the window reads,
+        // which need the state's head, then hit in L1
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(Q));
+        asm volatile("prefetch.global.L1 [%0];" ::"l"(Q + (w - 1)));
         UnitState s = p.state[b];
         double g, d;
         if (!isfinite(n)) {
@@ -282,8 +288,6 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
             g = CUDART_INF;
             d = CUDART_INF;
         } else {
-            const int w = p.window;
-            double *Q = p.queue + static_cast<int64_t>(b) * w;
             g = (s.count == 0 || s.mean == 0.0) ? 1.0 : n / (s.mean + p.eps);
             if (s.fill == w) {
                 // mean of the window, summed oldest to newest; loads issued 8 at a time
@@ -387,6 +391,17 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
     }
 }
 
+// Ticket increment with acquire-release semantics at GPU scope: it publishes
+// the caller's earlier writes (and, after a barrier, those of its CTA) and,
+// for the caller that draws the last ticket, makes every earlier holder's
+// writes visible.
+__device__ __forceinline__ uint32_t ticket_acq_rel(uint32_t *t)
+{
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(t) : "memory");
+    return old;
+}
+
 // A unit split over several warps: stores this warp's partial and takes a
 // ticket.  Returns true (with the unit's total in s) for the warp that takes
 // the last ticket; that warp sums the partials in slot order.
@@ -397,13 +412,12 @@ __device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, in
     uint32_t last = 0;
     if (lane == 0) {
         __stcg(&p.partial[base + (warp - p.first_warp[b])], s);
-        __threadfence();
-        last = atomicAdd(&p.unit_ticket[b], 1u) == static_cast<uint32_t>(parts - 1);
+        last = ticket_acq_rel(&p.unit_ticket[b]) == static_cast<uint32_t>(parts - 1);
     }
     last = __shfl_sync(kFull, last, 0);
     if (!last)
         return false;
-    __threadfence();
+    __syncwarp();                                    // lane 0's acquire orders the lanes' loads
     double acc = 0.0;
     for (int32_t j = lane; j < parts; j += 32)
         acc += __ldcg(&p.partial[base + j]);
@@ -875,14 +889,15 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     if (MODE == kStepPartials)
         return;
 
-    // Grid completion: the last CTA through runs the selection.
-    __threadfence();
+    // Grid completion: the last CTA through runs the selection.  The barrier
+    // orders the CTA's writes before thread 0's release; the last ticket's
+    // acquire, then the barrier, orders the selecting CTA's reads after
+    // every CTA's writes.
     __syncthreads();
     if (threadIdx.x == 0)
-        s_misc[0] = atomicAdd(&p.ctl->ctas_done, 1u) == gridDim.x - 1 ? 1u : 0u;
+        s_misc[0] = ticket_acq_rel(&p.ctl->ctas_done) == gridDim.x - 1 ? 1u : 0u;
     __syncthreads();
     if (s_misc[0]) {
-        __threadfence();
         select_and_commit(p, __ldcg(&p.ctl->steps) + 1, s_hist, s_misc, s_red, s_keys);
     }
 }
