@@ -14,9 +14,13 @@
 //
 // One warp per token row: pass 1 reads the row for amax (integer max over the
 // magnitude bits), pass 2 reads it again from L2 and writes the result, so
-// HBM sees one read and one write per element.  The grid holds 32 warps per
-// SM, whose rows (tens of MB in all) stay resident in the 129 MB L2 between
-// the two passes.  No shared memory, no block barrier, no waits.
+// HBM sees one read and one write per element.  The grid holds 16 warps per
+// SM, whose rows (about 30 MB in all) stay resident in the 129 MB L2 between
+// the two passes: pass 1 loads them with an L2 evict-last policy, pass 2
+// reads and the output stores use evict-first, so the write stream does not
+// push the waiting rows out.  (32 warps per SM left a fifth of the pass-2
+// reads missing L2; 8 cannot keep enough loads in flight.)  No shared memory,
+// no block barrier, no waits.
 #include <algorithm>
 #include <cmath>
 #include <cstdint>
@@ -50,7 +54,7 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kMinCtas = 4;             // 32 resident warps per SM: their rows stay in L2
+constexpr int kMinCtas = 2;             // 16 resident warps per SM: their rows stay in L2
 
 struct FqFmt {
     float fmax;
@@ -238,10 +242,38 @@ __device__ __forceinline__ RowRef locate_row(int64_t r, const void *in, void *ou
     return q;
 }
 
-// 16-byte load through L2 that stays in L2 for the second pass, and one that
-// is the last use.
-__device__ __forceinline__ uint4 ld_keep(const uint4 *p) { return __ldcg(p); }
-__device__ __forceinline__ uint4 ld_last(const uint4 *p) { return __ldcs(p); }
+// L2 eviction policies for a whole access (createpolicy), and 16-byte
+// accesses that carry one.
+__device__ __forceinline__ uint64_t policy_evict_last()
+{
+    uint64_t p;
+    asm("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_first()
+{
+    uint64_t p;
+    asm("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint4 ld_policy(const uint4 *q, uint64_t pol)
+{
+    uint4 r;
+    asm volatile("ld.global.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(q), "l"(pol));
+    return r;
+}
+__device__ __forceinline__ void st_policy(uint4 *q, uint4 v, uint64_t pol)
+{
+    asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;"
+                 ::"l"(q), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol) : "memory");
+}
+
+// Pass 1's load keeps the line in L2 for pass 2; pass 2's load is its last
+// use, and the output is written once.
+__device__ __forceinline__ uint4 ld_keep(const uint4 *p) { return ld_policy(p, policy_evict_last()); }
+__device__ __forceinline__ uint4 ld_last(const uint4 *p) { return ld_policy(p, policy_evict_first()); }
+__device__ __forceinline__ void st_once(uint4 *p, uint4 v) { st_policy(p, v, policy_evict_first()); }
 
 // Pass 2 of one row in format CODE (one warp): quantize and write.
 template <int DT, int CODE>
@@ -259,18 +291,18 @@ __device__ __forceinline__ void quantize_row_warp(const char *src, char *dst, co
             v[j] = ld_last(vs + i + j * 32);
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-            __stcs(vd + i + j * 32, quantize_vec<DT, CODE>(v[j], inv, scale));
+            st_once(vd + i + j * 32, quantize_vec<DT, CODE>(v[j], inv, scale));
     }
     for (; i < nvec; i += 32)
-        __stcs(vd + i, quantize_vec<DT, CODE>(ld_last(vs + i), inv, scale));
+        st_once(vd + i, quantize_vec<DT, CODE>(ld_last(vs + i), inv, scale));
     for (int64_t t = tail_at + lane; t < n; t += 32)
         Act<DT>::store(dst, t, fq_round2<CODE>(Act<DT>::load(src, t) * inv, 0.f).x * scale);
 }
 
 // One warp per token row, rows assigned round-robin.  Pass 1 reads the row
 // (8 16-byte loads in flight per lane) for amax; pass 2 reads it again -- from
-// L2, the resident warps' rows fit there -- and writes the result with
-// streaming stores.  No shared memory and no block barrier.
+// L2, the resident warps' rows fit there -- and writes the result once.  No
+// shared memory and no block barrier.
 template <int DT>
 __global__ void __launch_bounds__(kThreads, kMinCtas) fake_quant_kernel(
     const void *in, void *out, const int64_t *offset, const int64_t *cols, const int64_t *row_start,
@@ -311,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, kMinCtas) fake_quant_kernel(
                 for (int64_t t = lane; t < q.head; t += 32)
                     Act<DT>::copy(q.src, q.dst, t);
                 for (int64_t t = lane; t < q.nvec; t += 32)
-                    __stcs(vd + t, ld_last(vs + t));
+                    st_once(vd + t, ld_last(vs + t));
                 for (int64_t t = q.tail_at + lane; t < q.n; t += 32)
                     Act<DT>::copy(q.src, q.dst, t);
             }
