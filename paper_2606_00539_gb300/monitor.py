@@ -2,6 +2,7 @@
 the CUDA stream; every step of the monitor runs in libgnmr's kernel."""
 from __future__ import annotations
 
+import ctypes
 import math
 
 import numpy as np
@@ -174,6 +175,35 @@ class Monitor:
         if stream is None:
             stream = torch.cuda.current_stream(device)
         return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+    def prepare_step(self, arena, mask=None, stats: dict | None = None, stream=None):
+        """Validates and marshals step()'s arguments once and returns a
+        callable that enqueues one step with them: each call is one C call
+        (for loops where the Python cost of step() would gap the GPU).  The
+        tensors' storage and the stream are fixed at preparation; their
+        contents may change between calls (e.g. the next step's gradients
+        written into the same arena).  The callable returns the mask."""
+        torch = _torch()
+        dev = self._check_arena(arena)
+        if mask is None:
+            mask = torch.empty(self.num_units, dtype=torch.uint8, device=dev)
+        self._check_tensor(mask, "mask", torch.uint8, self.num_units)
+        st = self._stats_struct(stats)
+        fn = N.load().gnmr_step
+        args = (self._h, arena.data_ptr(), int(arena.numel()), self._stream_handle(stream, dev),
+                mask.data_ptr(), ctypes.byref(st) if st is not None else None)
+        keep = (arena, mask, stats, st)            # storage the prepared call points into
+        handle = self._h
+
+        def run():
+            if self._h != handle:
+                raise ValueError("the monitor was closed")
+            status = fn(*args)
+            if status:
+                N._check(status, handle)
+            return keep[1]
+
+        return run
 
     def step_partials(self, arena, sumsq=None, stream=None):
         """First half of a sharded step: per-unit sums of squares of this

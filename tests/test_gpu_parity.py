@@ -428,6 +428,37 @@ def test_pinned_host_arena_is_read_in_place(config, shrink, cuda_device):
         m_host.close()
 
 
+def test_prepared_step_matches_step(cuda_device):
+    """Monitor.prepare_step: the prepared call gives bitwise the outputs of
+    step() on the same arena contents, follows new contents written into the
+    same storage, and refuses to run after close()."""
+    import torch
+    w = workloads.make("aq-stress", shrink=4, steps=5)
+    f = workloads.Filler(w, cuda_device)
+    arena = f.new_arena()
+    m_a, m_b = _monitor(w), _monitor(w)
+    s_a, s_b = m_a.new_stats(), m_b.new_stats()
+    mask_b = torch.empty(w.num_units, dtype=torch.uint8, device=cuda_device)
+    run = m_b.prepare_step(arena, mask=mask_b, stats=s_b)
+    try:
+        for t in range(w.steps):
+            f.fill(arena, t)
+            a = m_a.step(arena, stats=s_a)
+            b = run()
+            torch.cuda.synchronize()
+            assert b is mask_b and torch.equal(a, b), f"mask, step {t + 1}"
+            for k in s_a:
+                x, y = s_a[k], s_b[k]
+                if x.dtype == torch.float64:
+                    x, y = x.view(torch.int64), y.view(torch.int64)
+                assert torch.equal(x, y), f"{k}, step {t + 1}"
+    finally:
+        m_a.close()
+        m_b.close()
+    with pytest.raises(ValueError, match="closed"):
+        run()
+
+
 @pytest.mark.parametrize("shape", ["small", "large"])
 def test_deterministic_across_handles_and_runs(shape, cuda_device):
     import torch
