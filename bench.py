@@ -163,15 +163,27 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None}
 
 
-def profiled_traffic(kernel_source: str):
-    """DRAM bytes per launch from the committed ncu summary, or None once the
-    kernel source has changed since the counters were taken."""
+STEP_KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_00539_gb300", "csrc", f)
+                       for f in ("gnmr_kernels.cu", "gnmr_stream.cuh", "gnmr_internal.h")]
+
+
+def kernel_source_hash(paths) -> str:
+    """First 16 hex digits of the sha256 of the concatenated source files."""
     import hashlib
+    h = hashlib.sha256()
+    for path in paths:
+        with open(path, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(paths):
+    """DRAM bytes per launch from the committed ncu summary, or None once the
+    kernel's sources have changed since the counters were taken."""
     try:
         with open(os.path.join(ROOT, "profiles", "gnmr_step_kernel_traffic.json")) as f:
             rec = json.load(f)
-        with open(kernel_source, "rb") as f:
-            h = hashlib.sha256(f.read()).hexdigest()[:16]
+        h = kernel_source_hash(paths)
     except (OSError, ValueError):
         return None
     if rec.get("kernel_source_sha256_16") != h:
@@ -375,7 +387,7 @@ def run_gnmr(args):
     kern_ms = statistics.mean(per_ms)
     peak, peak_kind = measured_peaks()
     achieved = gbytes / (kern_ms / 1e3)
-    traffic = profiled_traffic(os.path.join(ROOT, "paper_2606_00539_gb300", "csrc", "gnmr_kernels.cu"))
+    traffic = profiled_traffic(STEP_KERNEL_SOURCES)
 
     # end to end through the public API with the step's input in pinned host
     # memory and its result read back to the host, every step inside the

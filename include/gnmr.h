@@ -334,7 +334,7 @@ gnmr_status gnmr_actuator_destroy(gnmr_actuator *a);
  * and therefore cannot hold a gnmr_handle.  Computes n_b = ||g_b||_2 for
  * every unit (the values gnmr_step writes to stats->norm) into d_norms, using
  * as scratch only a device array that lives in the library's static data:
- * about 11.5 MiB, reserved on every GPU that loads the library until the
+ * about 5.6 MiB, reserved on every GPU that loads the library until the
  * process exits.  No cudaMalloc, cudaFree or other allocating call is made.
  *
  * Arguments: d_arena (device, dtype elements, aligned to the element size;
@@ -344,10 +344,10 @@ gnmr_status gnmr_actuator_destroy(gnmr_actuator *a);
  * written), stream (cudaStream_t as void*, NULL = legacy default stream).
  * Runs on the calling thread's current device.
  *
- * Limits: num_units <= 131072 and sum over units of max(1, ceil(length
- * bytes / 64 KiB)) <= 1048576 (so up to 64 GiB of gradient in large units);
- * beyond them GNMR_ERR_INVALID_ARG, with gnmr_last_error(NULL) reading
- * "units > 131072" or "chunks>1048576".  A unit outside [0, arena_elems)
+ * Limit: num_units <= 131072 (any arena size); beyond it
+ * GNMR_ERR_INVALID_ARG, with gnmr_last_error(NULL) reading "units > 131072".
+ * The arena is read as 64 KiB chunks split into contiguous ranges over the
+ * GPU's warps, at the step kernel's streaming rate.  A unit outside [0, arena_elems)
  * gives GNMR_ERR_LAYOUT ("unit off arena"); other details: "dtype unknown",
  * "NULL pointer", "arena misalign", "CUDA failed".  The call makes no host
  * allocation either, on success or failure.

@@ -1,0 +1,35 @@
+"""CPU checks of bench.py's bookkeeping: argument rules and the source hash
+that keys the committed DRAM-traffic record."""
+import json
+import os
+
+import pytest
+
+import bench
+
+
+def test_graph_and_flush_do_not_combine():
+    with pytest.raises(SystemExit):
+        bench.parse_args(["--graph", "--flush-l2"])
+    assert bench.parse_args(["--graph"]).graph
+
+
+def test_traffic_record_follows_the_step_kernel_sources(tmp_path, monkeypatch):
+    srcs = [tmp_path / "a.cu", tmp_path / "b.cuh"]
+    for i, p in enumerate(srcs):
+        p.write_text(f"// source {i}\n")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    rec = {"kernel_source_sha256_16": bench.kernel_source_hash(srcs), "traffic_bytes_per_launch": 123}
+    (prof / "gnmr_step_kernel_traffic.json").write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.profiled_traffic(srcs) == 123
+    srcs[1].write_text("// changed\n")
+    assert bench.profiled_traffic(srcs) is None
+
+
+def test_committed_traffic_record_names_a_hash():
+    with open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "profiles",
+                           "gnmr_step_kernel_traffic.json")) as f:
+        rec = json.load(f)
+    assert len(rec["kernel_source_sha256_16"]) == 16 and rec["traffic_bytes_per_launch"] > 25_375_539_200
