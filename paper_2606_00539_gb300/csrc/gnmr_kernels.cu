@@ -394,36 +394,97 @@ __device__ __forceinline__ void commit_selected(const StepParams &p, bool stat, 
 // The selecting CTA's copy of the candidates' risk keys: candidate i's
 // risk_key in keys[i] and whether it belongs to the capped pool in bit i of
 // pool_bits (the candidates outside it -- retained under the admission cap --
-// are selected without ranking).  One read of the candidate list fills it;
-// the radix passes then run on shared memory.
-constexpr uint32_t kKeyCache = 7168;
-constexpr size_t kKeyCacheBytes = sizeof(uint64_t) * kKeyCache + sizeof(uint32_t) * (kKeyCache / 32);
+// are selected without ranking), followed by the radix histogram.  One read
+// of the candidate list fills it; the radix passes then run on shared memory
+// with 11-bit digits (2048 bins), so a 64-bit key needs at most six passes
+// and risks that crowd into one octave usually resolve in three.
+constexpr int kWideBits = 11;
+constexpr int kWideBins = 1 << kWideBits;
+static_assert(kWideBins == 4 * kThreads, "four histogram bins per thread of the selecting CTA");
+constexpr uint32_t kKeyCache = 6144;
+constexpr size_t kKeyBitsOffset = sizeof(uint64_t) * kKeyCache;
+constexpr size_t kKeyHistOffset = kKeyBitsOffset + sizeof(uint32_t) * (kKeyCache / 32);
+constexpr size_t kKeyCacheBytes = kKeyHistOffset + sizeof(uint32_t) * kWideBins;
+static_assert(kKeyHistOffset % 16 == 0, "the histogram is read as 16-byte vectors");
 
 __device__ __forceinline__ bool in_pool(const uint32_t *pool_bits, uint32_t i)
 {
     return (pool_bits[i >> 5] >> (i & 31u)) & 1u;
 }
 
+// Bucket of the r-th largest digit in hist[kWideBins] (r >= 1), by the whole
+// CTA: thread t owns the four bins just below those of thread t - 1 (thread
+// 0 the highest); the counts above each thread's bins come from a warp scan
+// and a scan of the 16 warp totals (in wsum[16]).  misc[1] = the bucket,
+// misc[2] = r minus the count above it, misc[3] = its count.
+__device__ __forceinline__ void find_bucket_wide(const uint32_t *hist, uint32_t r, uint32_t *misc, uint32_t *wsum)
+{
+    const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
+    const int q4 = kWideBins / 4 - 1 - t;
+    const uint4 q = reinterpret_cast<const uint4 *>(hist)[q4];      // bins 4 q4 .. 4 q4 + 3
+    const uint32_t c4[4] = {q.w, q.z, q.y, q.x};                     // descending
+    const uint32_t sum = c4[0] + c4[1] + c4[2] + c4[3];
+    uint32_t incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t u = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o)
+            incl += u;
+    }
+    if (lane == 31)
+        wsum[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+        const uint32_t tot = lane < kWarpsPerCta ? wsum[lane] : 0u;
+        uint32_t x = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t u = __shfl_up_sync(kFull, x, o);
+            if (lane >= o)
+                x += u;
+        }
+        if (lane < kWarpsPerCta)
+            wsum[lane] = x - tot;                    // counts in the warps' higher bins
+    }
+    __syncthreads();
+    uint32_t above = wsum[wid] + incl - sum;
+    if (above < r && r <= above + sum) {             // exactly one thread
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (above + c4[j] >= r) {
+                misc[1] = static_cast<uint32_t>(4 * q4 + 3 - j);
+                misc[2] = r - above;
+                misc[3] = c4[j];
+                break;
+            }
+            above += c4[j];
+        }
+    }
+}
+
 // K-th largest (risk_key : index_key) among the pool's m <= kKeyCache cached
-// keys, 1 <= K < pool size: MSD radix select with 8-bit digits over the
+// keys, 1 <= K < pool size: MSD radix select with 11-bit digits over the
 // cached 64-bit keys, then, only if whole keys tie at the cut, over the unit
 // indices (read from the candidate list).  Exactly K pool keys compare >= the
 // returned threshold.  All threads of the CTA call this.
 __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K, const uint64_t *keys,
-                                    const uint32_t *pool_bits, uint32_t *hist, uint32_t *misc,
+                                    const uint32_t *pool_bits, uint32_t *hist, uint32_t *wsum, uint32_t *misc,
                                     uint64_t &thr_hi, uint32_t &thr_lo)
 {
     const int lo_bits = p.num_units > 1 ? 32 - __clz(static_cast<uint32_t>(p.num_units - 1)) : 0;
-    const int lo_digits = (lo_bits + 7) / 8;
     const uint32_t lane = threadIdx.x & 31u;
     uint64_t pre_hi = 0, msk_hi = 0;
     uint32_t pre_lo = 0, msk_lo = 0;
     uint32_t r = K;
-    for (int dgt = 0; dgt < 8 + lo_digits; ++dgt) {
-        const bool in_hi = dgt < 8;
-        const int shift = in_hi ? 56 - 8 * dgt : 8 * (lo_digits - 1 - (dgt - 8));
-        for (int i = threadIdx.x; i < 256; i += blockDim.x)
-            hist[i] = 0;
+    int pos_hi = 64, pos_lo = lo_bits;               // bits of each key part not yet decided
+    while (pos_hi > 0 || pos_lo > 0) {
+        const bool in_hi = pos_hi > 0;
+        int &pos = in_hi ? pos_hi : pos_lo;
+        const int width = pos < kWideBits ? pos : kWideBits;
+        pos -= width;
+        const int shift = pos;
+        const uint32_t dmask = (1u << width) - 1u;
+        reinterpret_cast<uint4 *>(hist)[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
         __syncthreads();
         // four keys per thread per iteration (independent chains)
         for (uint32_t w0 = threadIdx.x & ~31u; w0 < m; w0 += 4 * blockDim.x) {
@@ -438,11 +499,11 @@ __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K,
                     const uint64_t hi = keys[i];
                     take[j] = (hi & msk_hi) == pre_hi;
                     if (in_hi) {
-                        dig[j] = static_cast<uint32_t>(hi >> shift) & 0xffu;
+                        dig[j] = static_cast<uint32_t>(hi >> shift) & dmask;
                     } else if (take[j]) {           // whole keys tie: rank by unit index
                         const uint32_t lo = index_key(__ldcg(&p.cand[i].unit), p.num_units);
                         take[j] = (lo & msk_lo) == pre_lo;
-                        dig[j] = (lo >> shift) & 0xffu;
+                        dig[j] = (lo >> shift) & dmask;
                     }
                 }
             }
@@ -452,17 +513,17 @@ __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K,
                     atomicAdd(&hist[dig[j]], 1u);
         }
         __syncthreads();
-        find_bucket(hist, r, misc);
+        find_bucket_wide(hist, r, misc, wsum);
         __syncthreads();
         const uint32_t bucket = misc[1];
         const uint32_t in_bucket = misc[3];
         r = misc[2];
         if (in_hi) {
             pre_hi |= static_cast<uint64_t>(bucket) << shift;
-            msk_hi |= 0xffull << shift;
+            msk_hi |= static_cast<uint64_t>(dmask) << shift;
         } else {
             pre_lo |= bucket << shift;
-            msk_lo |= 0xffu << shift;
+            msk_lo |= dmask << shift;
         }
         __syncthreads();
         if (in_bucket == r)                          // every key with this prefix is in
@@ -515,7 +576,8 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
             }
         } else if (m <= kKeyCache) {
             uint64_t *keys = reinterpret_cast<uint64_t *>(key_cache);
-            uint32_t *pool_bits = reinterpret_cast<uint32_t *>(key_cache + sizeof(uint64_t) * kKeyCache);
+            uint32_t *pool_bits = reinterpret_cast<uint32_t *>(key_cache + kKeyBitsOffset);
+            uint32_t *wide_hist = reinterpret_cast<uint32_t *>(key_cache + kKeyHistOffset);
             const uint32_t lane = threadIdx.x & 31u;
             // one read of the candidate list (loads in flight per thread)
             for (uint32_t w0 = (threadIdx.x & ~31u); w0 < m; w0 += kSelectIlp * blockDim.x) {
@@ -542,7 +604,7 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
             __syncthreads();
             uint64_t thr_hi = 0;
             uint32_t thr_lo = 0;
-            radix_select_cached(p, m, K, keys, pool_bits, hist, misc, thr_hi, thr_lo);
+            radix_select_cached(p, m, K, keys, pool_bits, wide_hist, hist, misc, thr_hi, thr_lo);
             for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
                 bool sel;
                 if (!in_pool(pool_bits, i)) {
