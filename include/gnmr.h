@@ -353,10 +353,14 @@ gnmr_status gnmr_actuator_destroy(gnmr_actuator *a);
  * allocation either, on success or failure.
  *
  * The first call on a device looks up the array's device address for that
- * device; make that first call before any stream capture.  Every call shares
- * the one array and leaves its contents behind (each call clears what must
- * start at zero); calls that overlap on the GPU race on it, so callers must
- * serialise them (one stream, one thread at a time). */
+ * device; make that first call before any stream capture.  The layout tables
+ * are uploaded (pageable host->device copies) only when the layout, dtype or
+ * device differs from the previous call's; a call repeating the previous
+ * layout enqueues one memset and one kernel, so it may be captured in a CUDA
+ * graph.  Every call shares the one array and leaves its contents behind
+ * (each call clears what must start at zero); calls that overlap on the GPU
+ * race on it, so callers must serialise them (one stream, one thread at a
+ * time). */
 gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena_elems, int32_t dtype,
                                    int32_t num_units, const int64_t *offsets,
                                    const int64_t *lengths, double *d_norms, void *stream);
