@@ -110,3 +110,37 @@ def test_static_norms_follow_layout_changes(cuda_device):
     assert st == N.GNMR_OK
     torch.cuda.synchronize()
     np.testing.assert_allclose(out[:len(off)].cpu().numpy(), oracle.unit_norms(host, off, ln), rtol=RTOL, atol=0)
+
+
+def test_static_norms_repeat_layout_is_graph_capturable(cuda_device):
+    """Once a layout is on the device, a call repeating it enqueues no host
+    copies: it is captured in a CUDA graph, and replays compute the norms of
+    whatever the arena holds at replay time."""
+    import torch
+    import oracle
+    lib = N.load()
+    rng = np.random.default_rng(22)
+    n = 1 << 20
+    arena = torch.empty(n, dtype=torch.float32, device=cuda_device)
+    off = np.sort(rng.integers(0, n - 50_000, 64)).astype(np.int64)
+    ln = rng.integers(1, 50_000, 64).astype(np.int64)
+    out = torch.empty(64, dtype=torch.float64, device=cuda_device)
+    stream = torch.cuda.Stream(cuda_device)
+
+    def call():
+        return lib.gnmr_unit_norms_static(arena.data_ptr(), n, N.GNMR_DTYPE_F32, 64, off.ctypes.data,
+                                          ln.ctypes.data, out.data_ptr(), stream.cuda_stream)
+
+    arena.normal_()
+    assert call() == N.GNMR_OK                       # uploads the layout
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        assert call() == N.GNMR_OK
+    for scale in (0.5, 3.0):
+        host = (rng.standard_normal(n) * scale).astype(np.float32)
+        arena.copy_(torch.from_numpy(host))
+        torch.cuda.synchronize()
+        graph.replay()
+        torch.cuda.synchronize()
+        np.testing.assert_allclose(out.cpu().numpy(), oracle.unit_norms(host, off, ln), rtol=RTOL, atol=0)
