@@ -316,6 +316,22 @@ def test_nonfinite_gradients(cuda_device):
                      dict(window=3, max_o=2, lock_len=1, alpha=(1.5, 1.5), beta=(1.5, 1.5)), 9)
 
 
+@pytest.mark.parametrize("window", [1, 9, 13, 24])
+def test_window_lengths(window, cuda_device):
+    """Delta-GNMR windows outside the standard 5 and 8: a single entry, and
+    windows longer than the eight entries the epilogue reads per batch (the
+    ring wraps mid-batch and leaves a remainder); enough steps that every
+    window fills and wraps."""
+    rng = np.random.default_rng(100 + window)
+    U = 300
+    ln = rng.integers(1, 2000, U).astype(np.int64)
+    steps = window + 7
+    off, dev, make_step = _per_unit_levels_arena(rng, ln, steps, 0.3, cuda_device)
+    _parity_on_norms(off, ln, dev, make_step,
+                     dict(dtype="f32", window=window, max_o=6, lock_len=2, alpha=1.3, beta=1.2),
+                     dict(window=window, max_o=6, lock_len=2, alpha=(1.3, 1.3), beta=(1.2, 1.2)), steps)
+
+
 @pytest.mark.parametrize("max_o,lock_len,thr", [(0, 3, 1.05), (10_000, 0, 1.05), (7, 2, 0.9)])
 def test_budget_extremes_and_ties(max_o, lock_len, thr, cuda_device):
     """maxO = 0 (never select), maxO >= U (plain threshold), and thresholds
