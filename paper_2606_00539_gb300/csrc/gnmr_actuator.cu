@@ -55,6 +55,8 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMinCtas = 2;             // 16 resident warps per SM: their rows stay in L2
+constexpr int kPass1Loads = 16;         // 16-byte loads in flight per lane in pass 1 (from HBM)
+constexpr int kPass2Loads = 8;          // in pass 2 (from L2)
 
 struct FqFmt {
     float fmax;
@@ -284,13 +286,13 @@ __device__ __forceinline__ void quantize_row_warp(const char *src, char *dst, co
     for (int64_t i = lane; i < head; i += 32)
         Act<DT>::store(dst, i, fq_round2<CODE>(Act<DT>::load(src, i) * inv, 0.f).x * scale);
     int64_t i = lane;
-    for (; i + 3 * 32 < nvec; i += 4 * 32) {
-        uint4 v[4];
+    for (; i + (kPass2Loads - 1) * 32 < nvec; i += kPass2Loads * 32) {
+        uint4 v[kPass2Loads];
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
+        for (int j = 0; j < kPass2Loads; ++j)
             v[j] = ld_last(vs + i + j * 32);
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
+        for (int j = 0; j < kPass2Loads; ++j)
             st_once(vd + i + j * 32, quantize_vec<DT, CODE>(v[j], inv, scale));
     }
     for (; i < nvec; i += 32)
@@ -300,7 +302,7 @@ __device__ __forceinline__ void quantize_row_warp(const char *src, char *dst, co
 }
 
 // One warp per token row, rows assigned round-robin.  Pass 1 reads the row
-// (8 16-byte loads in flight per lane) for amax; pass 2 reads it again -- from
+// (16 16-byte loads in flight per lane) for amax; pass 2 reads it again -- from
 // L2, the resident warps' rows fit there -- and writes the result once.  No
 // shared memory and no block barrier.
 template <int DT>
@@ -321,13 +323,13 @@ __global__ void __launch_bounds__(kThreads, kMinCtas) fake_quant_kernel(
         for (int64_t i = lane; i < q.head; i += 32)
             mbits = max(mbits, elem_max_bits<DT>(q.src, i));
         int64_t i = lane;
-        for (; i + 7 * 32 < q.nvec; i += 8 * 32) {
-            uint4 v[8];
+        for (; i + (kPass1Loads - 1) * 32 < q.nvec; i += kPass1Loads * 32) {
+            uint4 v[kPass1Loads];
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
+            for (int j = 0; j < kPass1Loads; ++j)
                 v[j] = ld_keep(vs + i + j * 32);
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
+            for (int j = 0; j < kPass1Loads; ++j)
                 mbits = max(mbits, vec_max_bits<DT>(v[j]));
         }
         for (; i < q.nvec; i += 32)
