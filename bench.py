@@ -168,12 +168,18 @@ STEP_KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_00539_gb300", "csrc", f)
 
 
 def kernel_source_hash(paths) -> str:
-    """First 16 hex digits of the sha256 of the concatenated source files."""
+    """First 16 hex digits of the sha256 of the concatenated source files with
+    comments removed and whitespace collapsed: an edit to a comment leaves the
+    compiled kernel, and so its profile, unchanged."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for path in paths:
-        with open(path, "rb") as f:
-            h.update(f.read())
+        with open(path, encoding="utf-8") as f:
+            text = f.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
 
 

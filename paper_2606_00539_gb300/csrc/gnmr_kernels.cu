@@ -3,11 +3,11 @@
 // Phase 1, every warp (the hot loop).  Each warp owns one contiguous run of
 // the segment stream planned by gnmr_plan.cpp (a unit is one or more
 // segments of the arena).  For every segment piece in its run it streams the
-// gradient with 16-byte read-only loads (8 in flight per
-// lane, 4 KiB per warp per iteration), squares in fp32, sums blocks of 16
-// iterations in fp32 and the blocks in fp64, and all-reduces across the warp
-// with shuffles: n_b = ||g_b||_2 (Sec. 2, Eq. local_gradient).  No shared
-// memory, no block barrier on this path.
+// gradient with 16-byte read-only loads (8 or 16 in flight per lane, by the
+// loop shape), squares in fp32, sums blocks of 16 iterations in fp32 and the
+// blocks in fp64, and all-reduces across the warp with shuffles:
+// n_b = ||g_b||_2 (Sec. 2, Eq. local_gradient).  No shared memory, no block
+// barrier on this path.  (The streaming reduction lives in gnmr_stream.cuh.)
 //
 // Phase 2, the warp that completes unit b.  A unit split over several warps
 // collects their partial sums through fixed slots and a per-unit ticket; the
@@ -16,12 +16,14 @@
 // and run the unit epilogue 32 at a time, one unit per lane: Algorithm 1
 // (GNMR, Delta-GNMR, incremental mean, window queue), the combined risk
 // R = max{GNMR/alpha_t, Delta-GNMR/beta_t} and the candidate test
-// R > 1 or Lock > 0 (Sec. 3.3), appending candidates to a compact list.
+// R > 1 or Lock > 0 (Sec. 3.3), appending candidates to a compact list and
+// writing every unit's outcome if it is not selected.
 //
 // Phase 3, the last CTA to finish (grid ticket).  Top_maxO over the
 // candidate list by an in-CTA radix select on the 96-bit key
-// (R descending, unit index ascending), then the lock bookkeeping of
-// Algorithm 2, the mask write, and the reset of the counters for the next
+// (R descending, unit index ascending), run on a shared-memory copy of the
+// candidates' keys, then the lock bookkeeping of Algorithm 2 for the
+// selected units, the counts, and the reset of the counters for the next
 // launch.  No CTA ever waits for another: the tickets decide who continues,
 // so the kernel cannot hang whatever the grid size or residency.
 //

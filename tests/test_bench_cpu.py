@@ -17,14 +17,16 @@ def test_graph_and_flush_do_not_combine():
 def test_traffic_record_follows_the_step_kernel_sources(tmp_path, monkeypatch):
     srcs = [tmp_path / "a.cu", tmp_path / "b.cuh"]
     for i, p in enumerate(srcs):
-        p.write_text(f"// source {i}\n")
+        p.write_text(f"// source {i}\nint f{i}(int x) {{ return x + {i}; }}\n")
     prof = tmp_path / "profiles"
     prof.mkdir()
     rec = {"kernel_source_sha256_16": bench.kernel_source_hash(srcs), "traffic_bytes_per_launch": 123}
     (prof / "gnmr_step_kernel_traffic.json").write_text(json.dumps(rec))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     assert bench.profiled_traffic(srcs) == 123
-    srcs[1].write_text("// changed\n")
+    srcs[1].write_text("/* reworded */ // source 1, still\nint f1(int x)  {  return x + 1; }\n")
+    assert bench.profiled_traffic(srcs) == 123        # comments and spacing only
+    srcs[1].write_text("// source 1\nint f1(int x) { return x + 2; }\n")
     assert bench.profiled_traffic(srcs) is None
 
 
