@@ -41,8 +41,9 @@ def parse_args(argv=None):
     p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["gnmr", "reference"], default="gnmr")
-    p.add_argument("--kernel", choices=["step", "actuator"], default="step",
-                   help="step: the GNMR monitor (headline); actuator: the fake-quant actuator")
+    p.add_argument("--kernel", choices=["step", "actuator", "static-norms"], default="step",
+                   help="step: the GNMR monitor (headline); actuator: the fake-quant actuator; "
+                        "static-norms: the allocation-free per-unit norms entry point")
     p.add_argument("--tokens", type=int, default=4096, help="tokens per microbatch (actuator)")
     p.add_argument("--workload", default="llama2-13b")
     p.add_argument("--group", default="tensor", choices=["tensor", "block", "expert"],
@@ -571,6 +572,72 @@ def run_actuator(args):
     }), flush=True)
 
 
+def run_static_norms(args):
+    """gnmr_unit_norms_static on the workload's arena: per-unit norms with no
+    allocation.  The layout is uploaded by the first (warm-up) call; the timed
+    calls repeat it, as a training loop does.  Algorithmic bytes: the gradient
+    read once."""
+    import torch
+    import workloads
+    from paper_2606_00539_gb300 import _native as N
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = workloads.make(args.workload, shrink=args.shrink, group=args.group)
+    filler = workloads.Filler(w, dev)
+    arena = filler.new_arena()
+    filler.fill(arena, w.steps // 2)
+    out = torch.empty(w.num_units, dtype=torch.float64, device=dev)
+    off = np.ascontiguousarray(w.offsets, np.int64)
+    ln = np.ascontiguousarray(w.lengths, np.int64)
+    if w.segment_unit is not None:
+        raise SystemExit("static-norms times per-tensor units (--group tensor)")
+    dt = N.GNMR_DTYPE_BF16 if w.dtype == "bf16" else N.GNMR_DTYPE_F32
+    lib = N.load()
+    stream = torch.cuda.Stream(dev)
+
+    def call():
+        st = lib.gnmr_unit_norms_static(arena.data_ptr(), arena.numel(), dt, w.num_units, off.ctypes.data,
+                                        ln.ctypes.data, out.data_ptr(), stream.cuda_stream)
+        if st != N.GNMR_OK:
+            raise RuntimeError(f"gnmr_unit_norms_static: {N.status_string(st)}: {N.last_error(None)}")
+
+    for _ in range(max(1, args.warmup)):
+        call()
+    stream.synchronize()
+    sampler = ClockSampler(0)
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    torch.cuda.synchronize(dev)
+    wall0 = time.time()
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        call()
+        ev[i][1].record(stream)
+    stream.synchronize()
+    wall1 = time.time()
+    sampler.stop()
+    per_ms = [a.elapsed_time(b) for a, b in ev]
+    ms = statistics.mean(per_ms)
+    peak, peak_kind = measured_peaks()
+    gbs = w.grad_bytes / (ms / 1e3) / 1e9
+    print(json.dumps({
+        "metric": "GNMR allocation-free per-unit norms GB/s (gradient read once)",
+        "value": round(gbs, 2), "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": f"{w.name} ({w.num_units} units, {w.grad_elems} {w.dtype} elements"
+                               f"{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
+                   "l2": "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * 129e6 else "inputs fit in L2 (hot)"},
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(gbs / peak, 4), "traffic": None, "algorithmic_bytes": w.grad_bytes,
+                     "peak_source": f"{peak_kind} hbm_gbs", "kernel": f"static_norms_kernel<{w.dtype}>",
+                     "kernel_ms_min": round(min(per_ms), 4)},
+        "gpu_launches": args.steps, "clocks": sampler.summary(wall0, wall1),
+    }), flush=True)
+
+
 def _in_features(w):
     """Input width of every linear of a LLaMA layout (the saved activation of
     x @ W^T is [tokens, in_features])."""
@@ -588,6 +655,8 @@ def main(argv=None):
         run_reference(args)
     elif args.kernel == "actuator":
         run_actuator(args)
+    elif args.kernel == "static-norms":
+        run_static_norms(args)
     else:
         run_gnmr(args)
 
