@@ -59,6 +59,17 @@ def test_forced_warmup_parity(cuda_device):
     _run(w, dict(forced_recovery_steps=4), check=check)
 
 
+@pytest.mark.parametrize("policy", [dict(policy=1, forced_recovery_steps=1),
+                                    dict(policy=2, static_warmup_steps=1, static_fraction=0.1),
+                                    dict(policy=2, static_warmup_steps=0, static_fraction=0.1)])
+def test_short_warmups_parity(policy, cuda_device):
+    """One-step (and, for the static policy, empty) warm-ups: the all-on
+    step is the first step, and the static choice rests on one step's GNMR
+    (or on none: every sum 0, the lowest indices kept)."""
+    w = workloads.make("tiny", shrink=2, steps=12)
+    _run(w, policy)
+
+
 @pytest.mark.parametrize("seed", [0, 1])
 def test_static_top_fraction_parity(seed, cuda_device):
     w = workloads.make("llama2-13b", shrink=16, steps=14, seed=seed)

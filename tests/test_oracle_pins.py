@@ -408,15 +408,22 @@ def test_admission_cap_invariants(seed):
         lock_prev = res.lock.copy()
 
 
-def test_forced_and_static_policies():
+@pytest.mark.parametrize("n_forced,n_static", [(5, 6), (1, 1), (0, 0)])
+def test_forced_and_static_policies(n_forced, n_static):
+    """Forced warm-up: every recoverable unit selected for t <= n_forced.
+    Static policy: every recoverable unit selected for t <= n_static, then
+    the ceil(0.3 |B_rec|) largest GNMR sums over those steps (ties by index;
+    with no warm-up all sums are 0) for good.  A one-step warm-up is the
+    case where the all-on steps cannot lean on state left by an earlier
+    all-on step."""
     rng = np.random.default_rng(17)
     U, T = 20, 25
     rec = (rng.random(U) < 0.7).astype(np.uint8)
     tr = _spiky_trace(rng, T, U, spike_p=0.2)
     base = oracle.Controller(U, 3, 4, 2, recoverable=rec)
-    forced = oracle.Controller(U, 3, 4, 2, recoverable=rec, forced_recovery_steps=5)
+    forced = oracle.Controller(U, 3, 4, 2, recoverable=rec, forced_recovery_steps=n_forced)
     stat = oracle.Controller(U, 3, 4, 2, recoverable=rec, policy=oracle.POLICY_STATIC_TOP,
-                             static_warmup_steps=6, static_fraction=0.3)
+                             static_warmup_steps=n_static, static_fraction=0.3)
     gsum = np.zeros(U)
     fixed = None
     for t, norms in enumerate(tr, start=1):
@@ -424,9 +431,11 @@ def test_forced_and_static_policies():
         # the policies never change the statistics
         np.testing.assert_array_equal(rb.gnmr, rf.gnmr)
         np.testing.assert_array_equal(rb.gnmr, rs.gnmr)
-        if t <= 5:
+        if t <= n_forced:
             assert np.array_equal(rf.mask, rec) and rf.n_selected == rec.sum()
-        if t <= 6:
+        else:
+            np.testing.assert_array_equal(rf.risk, rb.risk)
+        if t <= n_static:
             assert np.array_equal(rs.mask, rec)
             gsum += np.where(rec == 1, rb.gnmr, 0.0)
         else:
