@@ -59,6 +59,8 @@ def parse_args(argv=None):
                    help="capture the K timed steps (K gnmr_step launches) in one CUDA graph and "
                         "replay it: no host gaps between steps")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-sparsity", action="store_true",
+                   help="skip the untimed pass over the trace that measures trigger sparsity")
     p.add_argument("--cpu-sample-units", type=int, default=0,
                    help="units in the CPU-oracle sample (0 = all: one full step)")
     p.add_argument("--ref-sample-units", type=int, default=42,
@@ -299,6 +301,48 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def exceedance_counts(gnmr, dgnmr, recoverable, alpha_t: float, beta_t: float):
+    """One step's contribution to the trigger-sparsity statistic of Table 3:
+    among the recoverable units, how many have GNMR > alpha_t and how many
+    Delta-GNMR > beta_t (the two thresholds of the combined risk, Sec. 3.3)."""
+    rec = np.asarray(recoverable) != 0
+    return (int(np.count_nonzero(rec & (np.asarray(gnmr) > alpha_t))),
+            int(np.count_nonzero(rec & (np.asarray(dgnmr) > beta_t))))
+
+
+def trigger_sparsity(w, filler, arena, dev) -> dict:
+    """Table 3's statistic on the workload's synthetic trace: a fresh monitor
+    runs steps 1..T of the trace (untimed, after the timed region) and the
+    share of (recoverable unit, step) pairs over each threshold is counted,
+    with the candidate and selected counts of Algorithm 2."""
+    import torch
+    from paper_2606_00539_gb300 import Monitor
+    mon = Monitor(w.offsets, w.lengths, device=dev.index, **w.monitor_kwargs())
+    stats = mon.new_stats()
+    mask = torch.empty(w.num_units, dtype=torch.uint8, device=dev)
+    rec = np.asarray(w.recoverable, np.uint8)
+    over_g = over_d = cand = sel = 0
+    try:
+        for t in range(w.steps):
+            filler.fill(arena, t)
+            mon.step(arena, mask=mask, stats=stats)
+            a_t = w.alpha[0] if t + 1 <= w.warmup_steps else w.alpha[1]
+            b_t = w.beta[0] if t + 1 <= w.warmup_steps else w.beta[1]
+            g, d = exceedance_counts(stats["gnmr"].cpu().numpy(), stats["dgnmr"].cpu().numpy(), rec, a_t, b_t)
+            c = stats["counts"].cpu().tolist()
+            over_g, over_d, cand, sel = over_g + g, over_d + d, cand + c[0], sel + c[1]
+    finally:
+        mon.close()
+    pairs = max(1, int(rec.sum()) * w.steps)
+    return {"gnmr_over_alpha_pct": round(100.0 * over_g / pairs, 4),
+            "dgnmr_over_beta_pct": round(100.0 * over_d / pairs, 4),
+            "candidates_per_step": round(cand / w.steps, 2),
+            "selected_per_step": round(sel / w.steps, 2),
+            "selected_pct": round(100.0 * sel / pairs, 4),
+            "steps": w.steps, "recoverable_units": int(rec.sum()),
+            "trace": "the workload's synthetic trace, steps 1..T, one fresh monitor, untimed"}
+
+
 # ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
@@ -462,6 +506,10 @@ def run_gnmr(args):
                           f"{sec:.2f} s wall on {threads} threads")}
     del host
 
+    sparsity = None
+    if rank == 0 and not args.no_sparsity:
+        sparsity = trigger_sparsity(w, filler, arenas[0], dev)
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": round(value, 3), "unit": "GB/s", "n_gpus": world,
@@ -496,6 +544,7 @@ def run_gnmr(args):
             "e2e_staged": e2e_staged,
             "gpu_launches": launches,
             "clocks": clocks,
+            "trigger_sparsity": sparsity,
         }
         print(json.dumps(line), flush=True)
     mon.close()

@@ -35,3 +35,14 @@ def test_committed_traffic_record_names_a_hash():
                            "gnmr_step_kernel_traffic.json")) as f:
         rec = json.load(f)
     assert len(rec["kernel_source_sha256_16"]) == 16 and rec["traffic_bytes_per_launch"] > 25_375_539_200
+
+
+def test_exceedance_counts_only_recoverable_units_strictly_over():
+    import numpy as np
+    g = np.array([1.5, 2.0, 0.9, 3.0, 1.1])
+    d = np.array([1.0, 1.6, 2.0, 1.5, 9.0])
+    rec = np.array([1, 1, 1, 1, 0], np.uint8)
+    # alpha = 1.5: units 1 and 3 (unit 0 equals it; unit 4 is not recoverable)
+    # beta = 1.5: units 1 and 2 (unit 3 equals it)
+    assert bench.exceedance_counts(g, d, rec, 1.5, 1.5) == (2, 2)
+    assert bench.exceedance_counts(g, d, np.zeros(5, np.uint8), 1.0, 1.0) == (0, 0)
