@@ -69,3 +69,64 @@ def test_sharded_norms_over_gloo():
     for r in (0, 1):
         np.testing.assert_allclose(got[r], want, rtol=1e-12, atol=0)
     assert np.array_equal(got[0], got[1])        # every rank sees the same sums
+
+
+def _controller_rank(rank, world, port, arenas, off, ln, q):
+    import torch
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    start, n = S.even_shards(len(arenas[0]), world)[rank]
+    lo, ll = S.shard_layout(off, ln, start, n)
+    ctl = oracle.Controller(len(off), window=3, max_o=2, lock_len=2, alpha=(1.5, 1.2), beta=(1.4, 1.4),
+                            warmup_steps=2)
+    out = []
+    try:
+        for arena in arenas:
+            local = arena[start:start + n].astype(np.float64)
+            t = torch.from_numpy(np.array([np.sum(local[o:o + k] ** 2) for o, k in zip(lo, ll)]))
+            dist.all_reduce(t, op=dist.ReduceOp.SUM)
+            res = ctl.step(np.sqrt(t.numpy()))
+            out.append((res.mask.copy(), res.lock.copy()))
+    finally:
+        ctl.close()
+    q.put((rank, out))
+    dist.destroy_process_group()
+
+
+def test_sharded_controller_gives_every_rank_the_same_decisions():
+    """The sharded step: each rank reduces its slice of every unit, the sums
+    are all-reduced, and every rank steps the same deterministic controller
+    (Algorithms 1-2) -- so the masks and locks agree across ranks and with an
+    unsharded controller on the whole arena."""
+    rng = np.random.default_rng(11)
+    off, ln = _layout(rng, 40)
+    total = int((off + ln).max()) + 7
+    scale = np.exp(rng.normal(0.0, 1.0, len(off)))
+    arenas = []
+    for t in range(8):
+        s = scale.copy()
+        s[rng.choice(len(off), 3, replace=False)] *= rng.uniform(5.0, 50.0, 3)   # spikes
+        a = np.zeros(total, np.float32)
+        for b, (o, k) in enumerate(zip(off, ln)):
+            a[o:o + k] = rng.standard_normal(k) * s[b]
+        arenas.append(a)
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    mp.start_processes(_controller_rank, args=(2, _free_port(), arenas, off, ln, q), nprocs=2,
+                       join=True, start_method="spawn")
+    got = dict(q.get(timeout=60) for _ in range(2))
+    ref = oracle.Controller(len(off), window=3, max_o=2, lock_len=2, alpha=(1.5, 1.2), beta=(1.4, 1.4),
+                            warmup_steps=2)
+    try:
+        selected = 0
+        for t, arena in enumerate(arenas):
+            res = ref.step(oracle.unit_norms(arena, off, ln))
+            selected += int(res.mask.sum())
+            for r in (0, 1):
+                assert np.array_equal(got[r][t][0], got[0][t][0]) and np.array_equal(got[r][t][1], got[0][t][1])
+                assert np.array_equal(got[r][t][0], res.mask), f"step {t + 1}, rank {r}: mask"
+                assert np.array_equal(got[r][t][1], res.lock), f"step {t + 1}, rank {r}: lock"
+        assert selected > 0                          # the spikes were selected at some step
+    finally:
+        ref.close()
