@@ -449,10 +449,20 @@ def run_gnmr(args):
     e2e_staged = None
     host = None
     if not args.no_e2e and args.e2e_steps > 0:
+        why = None
         try:
             host = torch.empty(arenas[0].numel(), dtype=arenas[0].dtype, pin_memory=True)
             host.copy_(arenas[0])
             host_mask = torch.empty(w.num_units, dtype=torch.uint8, pin_memory=True)
+        except RuntimeError as exc:
+            why = str(exc).splitlines()[0]
+            host = None
+        # every rank takes the same branch: the timed loops below hold collectives
+        if max_over_ranks(0.0 if why is None else 1.0, world, dev) > 0.0:
+            e2e = {"value": None, "unit": "GB/s",
+                   "error": why or "pinned host allocation failed on another rank"}
+            host = None
+        else:
             dst = arenas[-1]
             h2d = int(host.numel() * host.element_size())
 
@@ -471,24 +481,26 @@ def run_gnmr(args):
                 stream.synchronize()
                 return max_over_ranks(e0.elapsed_time(e1) / args.e2e_steps, world, dev)
 
-            ms = timed(lambda: mon.step(host, mask=mask, stream=stream))
-            e2e = {"value": round(world * gbytes / (ms / 1e3), 3), "unit": "GB/s",
-                   "ms_per_step": round(ms, 3), "h2d_bytes_per_step": h2d,
-                   "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
-                   "path": "gnmr_step reading the pinned host arena in place, mask -> pinned host"}
-
             def staged():
                 dst.copy_(host, non_blocking=True)
                 mon.step(dst, mask=mask, stream=stream)
 
-            ms = timed(staged)
-            e2e_staged = {"value": round(world * gbytes / (ms / 1e3), 3), "unit": "GB/s",
-                          "ms_per_step": round(ms, 3), "h2d_bytes_per_step": h2d,
-                          "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
-                          "path": "pinned host arena -> device copy, gnmr_step, mask -> pinned host"}
-        except RuntimeError as exc:
-            e2e = {"value": None, "unit": "GB/s", "error": str(exc).splitlines()[0]}
-            host = None
+            try:
+                ms = timed(lambda: mon.step(host, mask=mask, stream=stream))
+                e2e = {"value": round(world * gbytes / (ms / 1e3), 3), "unit": "GB/s",
+                       "ms_per_step": round(ms, 3), "h2d_bytes_per_step": h2d,
+                       "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
+                       "path": "gnmr_step reading the pinned host arena in place, mask -> pinned host"}
+                ms = timed(staged)
+                e2e_staged = {"value": round(world * gbytes / (ms / 1e3), 3), "unit": "GB/s",
+                              "ms_per_step": round(ms, 3), "h2d_bytes_per_step": h2d,
+                              "d2h_bytes_per_step": int(w.num_units), "steps": args.e2e_steps,
+                              "path": "pinned host arena -> device copy, gnmr_step, mask -> pinned host"}
+            except RuntimeError as exc:
+                if world > 1:
+                    raise          # the other ranks wait in a collective: fail loudly, not hang
+                e2e = {"value": None, "unit": "GB/s", "error": str(exc).splitlines()[0]}
+                host = None
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
