@@ -4,10 +4,18 @@
 //
 // A warp reads a segment with 16-byte loads on the non-coherent path (no L1
 // allocation, 256-byte L2 prefetch), squares in fp32, sums short blocks in
-// fp32 and everything beyond in fp64, and flags segments whose fp32 squares
+// fp32 and the blocks as an unevaluated pair of floats (hi + lo, about 48
+// significant bits), reduces the pairs across the warp the same way, and
+// converts to fp64 once per segment.  It flags segments whose fp32 squares
 // may have lost accuracy (denormal or overflowing squares), which the caller
 // recomputes with exact fp64 squares.  Any element alignment: a scalar head
 // and tail around the 16-byte body.
+//
+// Why float pairs: on GB300 an fp64 add has a 64-cycle dependent latency and
+// the SM retires one fp64 warp-instruction every 20 cycles, shared by all its
+// warps.  A five-round fp64 shuffle reduction per segment held that pipe 40 %
+// of the time on layouts of many small units and stalled the streams; the
+// fp32 error-free additions run on the fp32 pipe.
 #ifndef GNMR_STREAM_CUH
 #define GNMR_STREAM_CUH
 
@@ -17,7 +25,7 @@ namespace gnmr {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kFlush = 16;   // main-loop iterations summed in fp32 before the fp64 add
+constexpr int kFlush = 16;   // main-loop iterations summed in fp32 before the pair add
 
 template <int DT> struct Elem;
 template <> struct Elem<0> {             // fp32
@@ -111,6 +119,42 @@ __device__ __forceinline__ double warp_allreduce_sum(double v)
     return v;
 }
 
+// Knuth's TwoSum: s + e == a + b exactly, s = fl(a + b), in any operand
+// order (fl(a + b) == fl(b + a), and e is the exact rounding error).
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e)
+{
+    s = __fadd_rn(a, b);
+    const float bb = __fadd_rn(s, -a);
+    e = __fadd_rn(__fadd_rn(a, -__fadd_rn(s, -bb)), __fadd_rn(b, -bb));
+}
+
+// (hi, lo) += x for an unevaluated pair hi + lo.
+__device__ __forceinline__ void pair_add(float &hi, float &lo, float x)
+{
+    float s, e;
+    two_sum(hi, x, s, e);
+    hi = s;
+    lo = __fadd_rn(lo, e);
+}
+
+// Sum of the lanes' pairs (xor butterfly): both partners combine the same
+// two pairs with commutative operations, so every lane ends with the same
+// bits.  Returns hi + lo in fp64; hi_out = the pair's leading float.
+__device__ __forceinline__ double warp_allreduce_pair(float hi, float lo, float &hi_out)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ohi = __shfl_xor_sync(kFull, hi, o);
+        const float olo = __shfl_xor_sync(kFull, lo, o);
+        float s, e;
+        two_sum(hi, ohi, s, e);
+        hi = s;
+        lo = __fadd_rn(__fadd_rn(lo, olo), e);
+    }
+    hi_out = hi;
+    return static_cast<double>(hi) + static_cast<double>(lo);
+}
+
 // Sum of squares of n elements at seg, by the whole warp.  Returns the sum
 // in every lane and sets `suspect` when fp32 squaring may have lost accuracy:
 // a nonzero segment whose sum is below 2^-100 (denormal squares) or above
@@ -144,7 +188,7 @@ __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n,
     }
 
     const Vec *v = reinterpret_cast<const Vec *>(seg + head * kEB);
-    double acc = 0.0;
+    float acc_hi = 0.f, acc_lo = 0.f;
     int64_t i = lane;
     int cnt = 0;
     for (; i + (kUnroll - 1) * 32 < nvec; i += kUnroll * 32) {
@@ -165,7 +209,7 @@ __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n,
                 a[j] += a[j + w];
         blk += a[0];
         if (++cnt == kFlush) {
-            acc += static_cast<double>(blk);
+            pair_add(acc_hi, acc_lo, blk);
             blk = 0.f;
             cnt = 0;
         }
@@ -184,10 +228,11 @@ __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n,
         }
         blk += a;
     }
-    acc += static_cast<double>(blk);
-    acc = warp_allreduce_sum(acc);
+    pair_add(acc_hi, acc_lo, blk);
+    float lead;
+    const double acc = warp_allreduce_pair(acc_hi, acc_lo, lead);
     bits = __reduce_or_sync(kFull, bits);
-    suspect = (bits & Elem<DT>::kMagnitude) != 0u && !(acc >= 0x1p-100 && acc <= 0x1p+100);
+    suspect = (bits & Elem<DT>::kMagnitude) != 0u && !(lead >= 0x1p-100f && lead <= 0x1p+100f);
     return acc;
 }
 
