@@ -473,10 +473,12 @@ __device__ __forceinline__ void find_bucket_wide(const uint32_t *hist, uint32_t 
 // keys, 1 <= K < pool size: MSD radix select with 11-bit digits over the
 // cached 64-bit keys, then, only if whole keys tie at the cut, over the unit
 // indices (read from the candidate list).  Exactly K pool keys compare >= the
-// returned threshold.  All threads of the CTA call this.
+// returned threshold.  whole_pool: every cached candidate belongs to the
+// pool (no admission cap), so pool_bits is not read.  All threads of the CTA
+// call this.
 __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K, const uint64_t *keys,
-                                    const uint32_t *pool_bits, uint32_t *hist, uint32_t *wsum, uint32_t *misc,
-                                    uint64_t &thr_hi, uint32_t &thr_lo)
+                                    const uint32_t *pool_bits, bool whole_pool, uint32_t *hist, uint32_t *wsum,
+                                    uint32_t *misc, uint64_t &thr_hi, uint32_t &thr_lo)
 {
     const int lo_bits = p.num_units > 1 ? 32 - __clz(static_cast<uint32_t>(p.num_units - 1)) : 0;
     const uint32_t lane = threadIdx.x & 31u;
@@ -500,7 +502,7 @@ __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K,
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const uint32_t i = w0 + j * blockDim.x + lane;
-                take[j] = i < m && in_pool(pool_bits, i);
+                take[j] = i < m && (whole_pool || in_pool(pool_bits, i));
                 dig[j] = 0;
                 if (take[j]) {
                     const uint64_t hi = keys[i];
@@ -611,10 +613,10 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
             __syncthreads();
             uint64_t thr_hi = 0;
             uint32_t thr_lo = 0;
-            radix_select_cached(p, m, K, keys, pool_bits, wide_hist, hist, misc, thr_hi, thr_lo);
+            radix_select_cached(p, m, K, keys, pool_bits, !admission, wide_hist, hist, misc, thr_hi, thr_lo);
             for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
                 bool sel;
-                if (!in_pool(pool_bits, i)) {
+                if (admission && !in_pool(pool_bits, i)) {
                     sel = true;                              // retained outside the cap
                 } else {
                     const uint64_t key = keys[i];
