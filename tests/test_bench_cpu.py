@@ -46,3 +46,23 @@ def test_exceedance_counts_only_recoverable_units_strictly_over():
     # beta = 1.5: units 1 and 2 (unit 3 equals it)
     assert bench.exceedance_counts(g, d, rec, 1.5, 1.5) == (2, 2)
     assert bench.exceedance_counts(g, d, np.zeros(5, np.uint8), 1.0, 1.0) == (0, 0)
+
+
+def test_reference_arm_prints_the_contract_line(capsys):
+    """The reference arm (the oracle on the host cores) prints one JSON line
+    with the contract's keys; its e2e moves no bytes across the host link."""
+    bench.main(["--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "1",
+                "--ref-sample-units", "8"])
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC
+    assert line["value"] > 0 and line["unit"] == "GB/s" and line["higher_is_better"] is True
+    for key in ("n_gpus", "steps", "warmup", "ms_per_step", "scaling", "vs_baseline", "dtype",
+                "data", "config"):
+        assert key in line, key
+    assert line["vs_baseline"] is None and line["scaling"] == "weak"
+    cpu = line["cpu_baseline"]
+    assert cpu["kind"] == "oracle" and cpu["cores"] >= 1 and cpu["value"] == line["value"]
+    assert "units 0..7" in cpu["sample"]
+    e2e = line["e2e"]
+    assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
+    assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
