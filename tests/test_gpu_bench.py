@@ -1,0 +1,34 @@
+"""bench.py's GPU arm on a small workload: one JSON line with the keys the
+measurement contract names (roofline, CPU baseline, end-to-end leg, launch
+count, clocks), consistent with each other."""
+import json
+
+import pytest
+
+import bench
+
+pytestmark = pytest.mark.gpu
+
+
+def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
+    bench.main(["--workload", "tiny", "--steps", "4", "--warmup", "3", "--e2e-steps", "3"])
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["metric"] == bench.METRIC and line["unit"] == "GB/s" and line["value"] > 0
+    assert line["n_gpus"] == 1 and line["steps"] == 4 and line["warmup"] == 3
+    assert line["higher_is_better"] is True and line["scaling"] == "weak" and line["vs_baseline"] is None
+    assert line["dtype"] == "f32" and line["data"] == "synthetic" and "tiny" in line["config"]["workload"]
+    roof = line["roofline"]
+    assert roof["bound"] == "hbm" and roof["unit"] == "GB/s" and roof["peak"] > 0
+    assert roof["frac"] == pytest.approx(roof["achieved"] / roof["peak"], rel=1e-3)
+    assert roof["traffic"] is None                     # recorded for the 13B layout only
+    cpu = line["cpu_baseline"]
+    assert cpu["kind"] == "oracle" and cpu["value"] > 0 and cpu["cores"] >= 1 and cpu["sample"]
+    e2e = line["e2e"]
+    assert e2e["value"] > 0 and e2e["unit"] == "GB/s"
+    assert e2e["h2d_bytes_per_step"] >= line["config"]["bytes_per_step"]   # the whole arena, padding too
+    assert e2e["d2h_bytes_per_step"] > 0
+    assert line["gpu_launches"] == 4                   # one step kernel per timed step
+    clocks = line["clocks"]
+    assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(clocks)
+    sparsity = line["trigger_sparsity"]
+    assert sparsity["steps"] > 0 and 0 <= sparsity["selected_pct"] <= 100
