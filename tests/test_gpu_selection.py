@@ -129,3 +129,63 @@ def test_static_policy_ranks_by_gnmr_sum(cuda_device):
     rng = np.random.default_rng(9)
     steps = [_spread(rng), rng.uniform(0.5, 2.0, U), rng.uniform(0.5, 2.0, U)]
     _drive(steps, policy=oracle.POLICY_STATIC_TOP, static_warmup_steps=2, static_fraction=0.01)
+
+
+def _random_sums(rng, U, t, prev):
+    """Per-unit sums of squares for one step: spread values with exact zeros,
+    exact repeats of the previous step (equal risks), a few spikes and, now
+    and then, an infinite sum (a non-finite gradient)."""
+    s = np.exp(rng.normal(0.0, 1.0, U))
+    kind = rng.random(U)
+    s[kind < 0.10] = 0.0
+    if prev is not None:
+        rep = kind > 0.85
+        s[rep] = prev[rep]
+    spikes = rng.random(U) < 0.05
+    s[spikes] *= rng.uniform(10.0, 1e4, int(spikes.sum()))
+    if t > 2 and rng.random() < 0.2:
+        s[rng.integers(0, U)] = np.inf
+    return s
+
+
+@pytest.mark.parametrize("seed", range(64))
+def test_random_small_controllers_agree_exactly(seed, cuda_device):
+    """Random small configurations through the controller half: the unit
+    count, window, maxO (0, below and above U), T_lock, policy, thresholds
+    (some below 1, so risks tie at t = 1) and eps vary; sums include zeros,
+    repeats and infinities.  The GPU and the oracle get the same n_b and run
+    the same IEEE fp64 operations, so R, masks, locks and counts agree bit
+    for bit at every step."""
+    import torch
+    rng = np.random.default_rng(1000 + seed)
+    U = int(rng.integers(1, 200))
+    policy = int(rng.integers(0, 3))
+    kw = dict(window=int(rng.integers(1, 10)), max_o=int(rng.choice([0, 1, 3, max(1, U // 4), U, U + 2])),
+              lock_len=int(rng.integers(0, 5)), eps=float(rng.choice([0.0, 1e-8])))
+    a = tuple(float(x) for x in rng.choice([0.9, 1.1, 1.5, 2.0], 2))
+    b = tuple(float(x) for x in rng.choice([0.8, 1.3, 1.5], 2))
+    warm = int(rng.integers(0, 4))
+    pol = dict(policy=policy, forced_recovery_steps=int(rng.integers(0, 3)) if policy != 2 else 0,
+               static_warmup_steps=int(rng.integers(0, 4)) if policy == 2 else 0,
+               static_fraction=float(rng.choice([0.1, 0.25, 0.5])))
+    rec = (rng.random(U) < 0.8).astype(np.uint8)
+    mon = Monitor(np.zeros(U, np.int64), np.zeros(U, np.int64), dtype="f32", device=0, alpha=a, beta=b,
+                  warmup_steps=warm, recoverable=rec, **kw, **pol)
+    ctl = oracle.Controller(U, alpha=a, beta=b, warmup_steps=warm, recoverable=rec, **kw, **pol)
+    stats = mon.new_stats()
+    mask = torch.empty(U, dtype=torch.uint8, device="cuda:0")
+    prev = None
+    try:
+        for t in range(12):
+            sumsq = _random_sums(rng, U, t, prev)
+            prev = sumsq
+            mon.finish(torch.from_numpy(sumsq).to("cuda:0"), mask=mask, stats=stats)
+            want = ctl.step(np.sqrt(sumsq))
+            got_r = stats["risk"].cpu().numpy()
+            assert np.array_equal(got_r.view(np.uint64), want.risk.view(np.uint64)), f"step {t + 1}: R"
+            assert np.array_equal(mask.cpu().numpy(), want.mask), f"step {t + 1}: mask"
+            assert np.array_equal(stats["lock"].cpu().numpy(), want.lock), f"step {t + 1}: lock"
+            assert stats["counts"].cpu().tolist() == [want.n_candidates, want.n_selected], f"step {t + 1}: counts"
+    finally:
+        mon.close()
+        ctl.close()
