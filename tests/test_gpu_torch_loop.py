@@ -1,6 +1,7 @@
 """The monitor and the actuator inside a real PyTorch training loop.
 
-A small MLP's parameter gradients live in one flat fp32 arena (every
+A small MLP's parameter gradients (fp32, or bf16 for a bf16 model) live in
+one flat arena (every
 `.grad` is a view of it, so backward writes straight into the arena); each
 Linear's weight and bias form one block-level unit.  Every step: the
 monitor's norms against torch's own norms of the same gradients, its
@@ -31,25 +32,29 @@ def _has_margin(res, max_o, rel=1e-4):
     return True
 
 
-def test_training_loop_with_monitor_and_actuator(cuda_device):
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_training_loop_with_monitor_and_actuator(dtype, cuda_device):
     import torch
     torch.manual_seed(0)
     dev = cuda_device
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    ebytes = 2 if dtype == "bf16" else 4
+    align = 16 // ebytes
     layers = [torch.nn.Linear(64, 96), torch.nn.Linear(96, 96), torch.nn.Linear(96, 96), torch.nn.Linear(96, 10)]
     model = torch.nn.Sequential(layers[0], torch.nn.ReLU(), layers[1], torch.nn.ReLU(),
-                                layers[2], torch.nn.ReLU(), layers[3]).to(dev)
+                                layers[2], torch.nn.ReLU(), layers[3]).to(dev, tdt)
     params = list(model.parameters())                 # w0, b0, w1, b1, ...
     offs, lens, seg_unit, pos = [], [], [], 0
     for i, p in enumerate(params):
         offs.append(pos)
         lens.append(p.numel())
         seg_unit.append(i // 2)                       # a layer's weight and bias: one unit
-        pos += (p.numel() + 3) // 4 * 4               # 16-byte aligned starts
-    arena = torch.zeros(pos, dtype=torch.float32, device=dev)
+        pos += (p.numel() + align - 1) // align * align   # 16-byte aligned starts
+    arena = torch.zeros(pos, dtype=tdt, device=dev)
     for p, o in zip(params, offs):
         p.grad = arena[o:o + p.numel()].view_as(p)
     U = len(layers)
-    mon = Monitor(np.array(offs, np.int64), np.array(lens, np.int64), dtype="f32", device=0,
+    mon = Monitor(np.array(offs, np.int64), np.array(lens, np.int64), dtype=dtype, device=0,
                   segment_unit=np.array(seg_unit, np.int32), num_units=U, alpha=ALPHA, beta=BETA, **KW)
     ctl = oracle.Controller(U, alpha=ALPHA, beta=BETA, **KW)
     stats = mon.new_stats()
@@ -60,10 +65,11 @@ def test_training_loop_with_monitor_and_actuator(cuda_device):
     rows = 256
     cols = np.array([l.in_features for l in layers], np.int64)
     a_off = np.concatenate([[0], np.cumsum(rows * cols)[:-1]]).astype(np.int64)
-    act = N.gnmr_actuator_create(a_off, np.full(U, rows, np.int64), cols, N.GNMR_DTYPE_F32, 0)
+    act = N.gnmr_actuator_create(a_off, np.full(U, rows, np.int64), cols,
+                                 N.GNMR_DTYPE_BF16 if dtype == "bf16" else N.GNMR_DTYPE_F32, 0)
     opt = torch.optim.SGD(model.parameters(), lr=0.05)
     gen = torch.Generator().manual_seed(1)
-    X = torch.randn(rows, 64, generator=gen).to(dev)
+    X = torch.randn(rows, 64, generator=gen).to(dev, tdt)
     Y = torch.randint(0, 10, (rows,), generator=gen).to(dev)
     compared = selected = 0
     try:
@@ -72,7 +78,7 @@ def test_training_loop_with_monitor_and_actuator(cuda_device):
             arena.zero_()
             loss = torch.nn.functional.cross_entropy(model(xb), Y)
             loss.backward()
-            assert all(p.grad.data_ptr() == arena.data_ptr() + 4 * o for p, o in zip(params, offs))
+            assert all(p.grad.data_ptr() == arena.data_ptr() + ebytes * o for p, o in zip(params, offs))
             mask = mon.step(arena, stats=stats)
             want_n = np.array([np.sqrt(sum(float(params[j].grad.double().pow(2).sum()) for j in (2 * u, 2 * u + 1)))
                                for u in range(U)])
@@ -90,12 +96,14 @@ def test_training_loop_with_monitor_and_actuator(cuda_device):
             a_out = torch.empty_like(a_in)
             N.gnmr_actuator_apply(act, a_in.data_ptr(), a_out.data_ptr(), a_in.numel(), mask.data_ptr(),
                                   N.GNMR_FQ_E2M1, N.GNMR_FQ_E4M3)
-            host_in, host_out = a_in.cpu().numpy(), a_out.cpu().numpy()
+            bits = (lambda t: t.cpu().view(torch.int16).numpy().view(np.uint16)) if dtype == "bf16" \
+                else (lambda t: t.cpu().numpy())
+            host_in, host_out = bits(a_in), bits(a_out)
             for u in range(U):
                 blk = slice(int(a_off[u]), int(a_off[u] + rows * cols[u]))
                 code = N.GNMR_FQ_E4M3 if got_mask[u] else N.GNMR_FQ_E2M1
                 want = oracle.fake_quant(host_in[blk].reshape(rows, int(cols[u])), code)
-                assert np.array_equal(host_out[blk].view(np.uint32), want.reshape(-1).view(np.uint32)), \
+                assert np.array_equal(host_out[blk].view(np.uint8), want.reshape(-1).view(np.uint8)), \
                     f"step {step + 1}, unit {u}: actuator"
             opt.step()
     finally:
