@@ -33,3 +33,18 @@ def shard_layout(offsets, lengths, shard_start: int, shard_elems: int):
     local_len = np.maximum(hi - lo, 0)
     local_off = np.where(local_len > 0, lo - shard_start, 0)
     return local_off.astype(np.int64), local_len.astype(np.int64)
+
+
+def sharded_step(mon, local_arena, *, group=None, sumsq=None, mask=None, stats=None):
+    """One step of the sharded path for a rank whose gradient shard is
+    `local_arena` (a handle created with the rank's `shard_layout`):
+    this rank's per-unit sums of squares (gnmr_step_partials), their sum over
+    the ranks of `group` (torch.distributed all-reduce, U fp64 values), then
+    Algorithms 1-2 on the summed sums (gnmr_finish).  Every rank passes the
+    same sums to the same deterministic controller, so every rank gets the
+    same mask.  All three run on torch's current stream, which the
+    all-reduce orders against.  Returns the mask tensor."""
+    import torch.distributed as dist
+    sums = mon.step_partials(local_arena, sumsq=sumsq)
+    dist.all_reduce(sums, op=dist.ReduceOp.SUM, group=group)
+    return mon.finish(sums, mask=mask, stats=stats)

@@ -148,3 +148,36 @@ def test_set_state_rejects_bad_blobs(cuda_device):
     finally:
         a.close()
         other.close()
+
+
+def test_sharded_step_helper_over_a_one_rank_nccl_group(cuda_device):
+    """sharding.sharded_step with a real process group (NCCL, one rank: the
+    shard is the whole arena and the all-reduce an identity) gives the
+    masks, locks and norms of a plain gnmr_step handle."""
+    import os
+    import socket
+    import torch
+    import torch.distributed as dist
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("nccl", rank=0, world_size=1, device_id=cuda_device)
+    w = workloads.make("tiny", steps=10)
+    f = workloads.Filler(w, cuda_device)
+    arena = f.new_arena()
+    plain, sharded = _monitor(w), _monitor(w)
+    sp, ss = plain.new_stats(), sharded.new_stats()
+    try:
+        for t in range(w.steps):
+            f.fill(arena, t)
+            m1 = plain.step(arena, stats=sp)
+            m2 = sharding.sharded_step(sharded, arena, stats=ss)
+            torch.cuda.synchronize()
+            assert torch.equal(m1, m2), f"step {t + 1}: mask"
+            assert torch.equal(sp["lock"], ss["lock"]), f"step {t + 1}: lock"
+            np.testing.assert_allclose(ss["norm"].cpu().numpy(), sp["norm"].cpu().numpy(), rtol=1e-12, atol=0)
+    finally:
+        plain.close()
+        sharded.close()
+        dist.destroy_process_group()

@@ -130,3 +130,51 @@ def test_sharded_controller_gives_every_rank_the_same_decisions():
         assert selected > 0                          # the spikes were selected at some step
     finally:
         ref.close()
+
+
+class _RecordingMonitor:
+    """Stands in for Monitor on CPU: its partial sums are the rank's local
+    sums of squares, and finish records what it was given."""
+
+    def __init__(self, arena, lo, ll):
+        self.arena, self.lo, self.ll = arena, lo, ll
+        self.finished = None
+
+    def step_partials(self, local_arena, sumsq=None):
+        import torch
+        local = local_arena.numpy().astype(np.float64)
+        return torch.tensor([np.sum(local[o:o + k] ** 2) for o, k in zip(self.lo, self.ll)],
+                            dtype=torch.float64)
+
+    def finish(self, sums, mask=None, stats=None):
+        self.finished = sums.numpy().copy()
+        return "mask"
+
+
+def _helper_rank(rank, world, port, arena, off, ln, q):
+    import torch
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    start, n = S.even_shards(len(arena), world)[rank]
+    lo, ll = S.shard_layout(off, ln, start, n)
+    mon = _RecordingMonitor(arena, lo, ll)
+    out = S.sharded_step(mon, torch.from_numpy(arena[start:start + n].copy()))
+    q.put((rank, out, mon.finished))
+    dist.destroy_process_group()
+
+
+def test_sharded_step_helper_finishes_on_the_summed_sums():
+    rng = np.random.default_rng(21)
+    off, ln = _layout(rng, 50)
+    arena = rng.standard_normal(int((off + ln).max()) + 3).astype(np.float32)
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    mp.start_processes(_helper_rank, args=(2, _free_port(), arena, off, ln, q), nprocs=2, join=True,
+                       start_method="spawn")
+    got = dict((r, (out, fin)) for r, out, fin in (q.get(timeout=60) for _ in range(2)))
+    want = oracle.unit_norms(arena, off, ln) ** 2
+    for r in (0, 1):
+        assert got[r][0] == "mask"
+        np.testing.assert_allclose(got[r][1], want, rtol=1e-12, atol=1e-300)
+    assert np.array_equal(got[0][1], got[1][1])
