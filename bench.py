@@ -33,6 +33,8 @@ if ROOT not in sys.path:
 
 METRIC = "GNMR step µs & grad GB/s (% HBM peak), LLaMA-2-13B 280-unit layout"
 FALLBACK_HBM_GBS = 6800.0
+PER_WORKLOADS = ("tiny", "llama2-1.3b", "llama2-13b", "moe", "aq-stress")
+L2_BYTES = 129e6
 
 
 def parse_args(argv=None):
@@ -63,8 +65,12 @@ def parse_args(argv=None):
                    help="skip the untimed pass over the trace that measures trigger sparsity")
     p.add_argument("--cpu-sample-units", type=int, default=0,
                    help="units in the CPU-oracle sample (0 = all: one full step)")
-    p.add_argument("--ref-sample-units", type=int, default=42,
-                   help="units per step of the reference arm (host-generated)")
+    p.add_argument("--ref-sample-units", type=int, default=0,
+                   help="units per step of the reference arm (0 = every unit: the full step)")
+    p.add_argument("--no-per-workload", action="store_true",
+                   help="skip the per-workload records (every workload's own trace steps)")
+    p.add_argument("--per-workload", default=",".join(PER_WORKLOADS),
+                   help="comma-separated workloads for the per-workload records")
     args = p.parse_args(argv)
     if args.graph and args.flush_l2:
         p.error("--graph times back-to-back steps; it does not combine with --flush-l2")
@@ -186,14 +192,15 @@ def kernel_source_hash(paths) -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(paths):
-    """DRAM bytes per launch from the committed ncu summary, or None once the
-    kernel's sources have changed since the counters were taken."""
+def profiled_traffic(paths, workload: str = "llama2-13b"):
+    """DRAM bytes per launch of `workload`'s step from the committed ncu
+    record, or None if there is none or the kernel's sources have changed
+    since its counters were taken."""
     try:
         with open(os.path.join(ROOT, "profiles", "gnmr_step_kernel_traffic.json")) as f:
-            rec = json.load(f)
+            rec = json.load(f)["records"][workload]
         h = kernel_source_hash(paths)
-    except (OSError, ValueError):
+    except (OSError, KeyError, TypeError, ValueError):
         return None
     if rec.get("kernel_source_sha256_16") != h:
         return None
@@ -221,13 +228,13 @@ def host_cores() -> int:
         return os.cpu_count() or 1
 
 
-def cpu_oracle_rate(view, w, units, reps: int = 1):
+def cpu_oracle_rate(view, w, units, reps: int = 1, threads: int = 0):
     """Times the oracle (norms of `units` + Algorithms 1-2 over them) and
-    returns (GB/s, threads, seconds per rep)."""
+    returns (GB/s, threads, seconds per rep); threads = 0: every host core."""
     import oracle
     off = w.offsets[units]
     ln = w.lengths[units]
-    threads = min(host_cores(), len(units))
+    threads = min(threads or host_cores(), len(units))
     ctl = oracle.Controller(len(units), **dict(w.controller_kwargs(),
                                                recoverable=w.recoverable[units]))
     times = []
@@ -242,16 +249,77 @@ def cpu_oracle_rate(view, w, units, reps: int = 1):
     return nbytes / sec / 1e9, threads, sec
 
 
-def bf16_bits(x: np.ndarray) -> np.ndarray:
-    """float32 -> bfloat16 bit patterns, round to nearest even."""
-    u = x.astype(np.float32).view(np.uint32)
-    r = ((u >> 16) & 1) + 0x7FFF
-    return ((u + r) >> 16).astype(np.uint16)
+def workload_config(w, args, n_arenas: int, world: int) -> dict:
+    """The `config` object both arms print: what the workload is, not how a
+    kernel runs it (the same dict on the GPU arm and the reference arm)."""
+    return {"workload": f"{w.name} ({w.num_units} units, {w.num_segments} tensors, "
+                        f"{w.grad_elems} {w.dtype} "
+                        f"elements{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
+            "bytes_per_step": w.grad_bytes, "arenas_cycled": n_arenas,
+            "l2": ("L2 flushed before every step (512 MB write)" if getattr(args, "flush_l2", False)
+                   else "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * L2_BYTES
+                   else "inputs fit in L2 (hot)"),
+            "parallelism": "replicas" if world > 1 else "single GPU"}
 
 
 # ---------------------------------------------------------------------------
 # reference arm: the oracle on the host cores
 # ---------------------------------------------------------------------------
+
+HOST_BLOCK = 1 << 24
+
+
+def host_arena(w, step: int, units, threads: int) -> np.ndarray:
+    """A host copy of one arena of workload `w` (same packing: w.offsets,
+    w.arena_elems) for the oracle, generated on the host cores without the
+    GPU.  One seeded N(0, 1) block of 16 Mi values is tiled over every unit
+    (starting at a unit-dependent position) and scaled by the power of two
+    nearest the unit's scale at trace step `step` (0-based), which for these
+    float formats is an exact integer add on the exponent field; a unit with
+    scale 0 (an unrouted expert) is all zeros.  The oracle's cost does not
+    depend on the values, only on the layout."""
+    from concurrent.futures import ThreadPoolExecutor
+    rng = np.random.default_rng([w.seed, 17, step])
+    block = rng.standard_normal(HOST_BLOCK, dtype=np.float32)
+    block[np.abs(block) < 1e-6] = 1e-6                       # keep every value normal
+    if w.dtype == "bf16":
+        u = block.view(np.uint32)
+        u += ((u >> 16) & 1) + 0x7FFF                          # round to nearest even
+        bits = (u >> 16).astype(np.uint16)
+        out = np.zeros(w.arena_elems, np.uint16)
+        shift, dt = 7, np.uint16
+    else:
+        bits = block.view(np.uint32).copy()
+        out = np.zeros(w.arena_elems, np.float32)
+        shift, dt = 23, np.uint32
+    view = out.view(dt)
+    scales = w.scales[step]
+
+    def one(s):
+        sc = float(scales[s])
+        if sc == 0.0:
+            return
+        k = int(round(math.log2(sc)))
+        off, n = int(w.offsets[s]), int(w.lengths[s])
+        start = (s * 7919) % HOST_BLOCK
+        pos = 0
+        while pos < n:
+            take = min(n - pos, HOST_BLOCK - start)
+            dst = view[off + pos:off + pos + take]
+            np.copyto(dst, bits[start:start + take])
+            # |k| is small (log-normal scales, spikes up to 10^4), so no
+            # exponent field over- or underflows
+            if k > 0:
+                np.add(dst, dt(k << shift), out=dst)
+            elif k < 0:
+                np.subtract(dst, dt(-k << shift), out=dst)
+            pos += take
+            start = 0
+
+    with ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
+        list(ex.map(one, [int(s) for s in units]))
+    return out
+
 
 def run_reference(args):
     rank, _, world = dist_env()
@@ -260,44 +328,45 @@ def run_reference(args):
     import oracle
     import workloads
     w = workloads.make(args.workload, shrink=args.shrink)
-    units = np.arange(min(args.ref_sample_units, w.num_units))
+    k = args.ref_sample_units or w.num_units
+    units = np.arange(min(k, w.num_units))
     off = w.offsets[units]
     ln = w.lengths[units]
-    rng = np.random.default_rng(0)
-    # host-generated sample arena (same unit sizes and scale model)
-    local_off = np.concatenate([[0], np.cumsum(ln)[:-1]]).astype(np.int64)
-    arena = np.empty(int(ln.sum()), dtype=np.uint16 if w.dtype == "bf16" else np.float32)
-    for i, u in enumerate(units):
-        z = (rng.standard_normal(int(ln[i])) * w.scales[0, u]).astype(np.float32)
-        arena[local_off[i]:local_off[i] + ln[i]] = bf16_bits(z) if w.dtype == "bf16" else z
     threads = min(host_cores(), len(units))
+    n_arenas = max(1, args.arenas)
+    # the trace steps the GPU arm cycles, generated on the host (untimed)
+    arenas = [host_arena(w, (w.steps // 2 + i) % w.steps, units, host_cores()) for i in range(n_arenas)]
     ctl = oracle.Controller(len(units), **dict(w.controller_kwargs(),
                                                recoverable=w.recoverable[units]))
-    for _ in range(args.warmup):
-        ctl.step(oracle.unit_norms_threaded(arena, local_off, ln, threads))
+    for i in range(args.warmup):
+        ctl.step(oracle.unit_norms_threaded(arenas[i % n_arenas], off, ln, threads))
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        ctl.step(oracle.unit_norms_threaded(arena, local_off, ln, threads))
+    for i in range(args.steps):
+        ctl.step(oracle.unit_norms_threaded(arenas[(args.warmup + i) % n_arenas], off, ln, threads))
     sec = (time.perf_counter() - t0) / max(args.steps, 1)
     ctl.close()
     nbytes = int(ln.sum()) * w.elem_bytes
     gbs = nbytes / sec / 1e9
-    sample = (f"units 0..{len(units) - 1} of the {w.num_units}-unit {w.name} layout "
-              f"({nbytes / 1e9:.3f} GB of {w.grad_bytes / 1e9:.3f} GB per step), host-generated")
+    full = len(units) == w.num_units
+    what = (f"every step the whole {w.num_units}-unit {w.name} layout" if full
+            else f"units 0..{len(units) - 1} of the {w.num_units}-unit {w.name} layout")
+    sample = (f"{what} ({nbytes / 1e9:.3f} GB of {w.grad_bytes / 1e9:.3f} GB per step): unit norms "
+              f"on {threads} threads (contiguous unit groups of equal bytes, each unit summed "
+              f"sequentially in double) + Algorithms 1-2; {n_arenas} host-generated arenas cycled")
     line = {
         "impl": "reference", "metric": METRIC, "value": round(gbs, 4), "unit": "GB/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(w.grad_bytes / (gbs * 1e9) * 1e3, 3),
+        "ms_per_step": round(nbytes / (gbs * 1e9) * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
         "data": "synthetic",
-        "config": {"workload": f"{w.name} ({w.num_units} units, {w.grad_elems} {w.dtype} elements)",
-                   "bytes_per_step": w.grad_bytes},
+        "config": workload_config(w, args, n_arenas, world),
         "cpu_baseline": {"value": round(gbs, 4), "unit": "GB/s", "cores": threads,
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(gbs, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
-        "note": "ms_per_step extrapolates the sample rate to the full step",
     }
+    if not full:
+        line["note"] = "a sample of the layout's units: value is the sample's GB/s"
     print(json.dumps(line), flush=True)
 
 
@@ -347,6 +416,187 @@ def trigger_sparsity(w, filler, arena, dev) -> dict:
 # the GPU arm
 # ---------------------------------------------------------------------------
 
+def trace_window(trace_steps: int, k: int, w: int):
+    """(first timed trace step, 1-based; number of timed steps): K steps in
+    the middle of the trace, after at least W warm-up steps."""
+    w = max(0, min(w, trace_steps - 1))
+    k = max(1, min(k, trace_steps - w))
+    t0 = max(w + 1, (trace_steps - k) // 2 + 1)
+    return t0, min(k, trace_steps - t0 + 1)
+
+
+def workload_record(name, k_steps, w_steps, dev, peak, sampler, budget_bytes):
+    """workload_record_on with every allocation, fill, step and event on one
+    stream, so their order is the order of the calls."""
+    import torch
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        return workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budget_bytes)
+
+
+def workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budget_bytes):
+    """One workload's timing on its own trace: a fresh monitor runs trace
+    steps 1..t0-1 (warm-up), its state is saved, and each timing pass
+    restores it and runs trace steps t0..t0+K-1, so every pass makes the
+    trace's own candidate pools and selections.  Arenas that fit in
+    `budget_bytes` are all generated first (passes: back-to-back prepared
+    calls with per-step events, one CUDA graph of the K calls, and, for
+    arenas under 2 GB, an L2 flush before every step); larger ones are
+    regenerated between steps, outside each step's events, followed by a
+    512 MB read so the step starts with no dirty or arena lines in L2."""
+    import torch
+    import workloads
+    from paper_2606_00539_gb300 import Monitor
+
+    w = workloads.make(name)
+    filler = workloads.Filler(w, dev)
+    t0, K = trace_window(w.steps, k_steps, w_steps)
+    mon = Monitor(w.offsets, w.lengths, device=dev.index, **w.monitor_kwargs())
+    info = mon.info()
+    stats = mon.new_stats()
+    counts = torch.zeros((K, 2), dtype=torch.int32, device=dev)
+    mask = torch.empty(w.num_units, dtype=torch.uint8, device=dev)
+    arena_bytes = w.arena_elems * w.elem_bytes
+    distinct = K * arena_bytes <= budget_bytes
+    rec = {"trace_steps": [t0, t0 + K - 1], "steps": K, "warmup_steps": t0 - 1,
+           "units": w.num_units, "dtype": w.dtype, "bytes_per_step": w.grad_bytes,
+           "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, {info['num_warps']} warp runs, "
+                   f"{'large-unit' if info['loop_shape'] == 2 else 'small-unit'} loop shape"}
+    def fill(arena, i):
+        filler.fill(arena, i)                       # on the current stream: `stream`
+
+    scratch = filler.new_arena()
+    for i in range(t0 - 1):                         # warm-up: trace steps 1..t0-1
+        fill(scratch, i)
+        mon.step(scratch, mask=mask, stats=stats, stream=stream)
+    blob = mon.get_state(stream)
+    step_stats = [dict(stats, counts=counts[j]) for j in range(K)]
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    region = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    per_pass_counts = []
+
+    def us(ms):
+        return round(ms * 1e3, 1)
+
+    if distinct:
+        del scratch
+        arenas = []
+        for j in range(K):
+            a = filler.new_arena()
+            fill(a, t0 - 1 + j)
+            arenas.append(a)
+        calls = [mon.prepare_step(arenas[j], mask=mask, stats=step_stats[j], stream=stream) for j in range(K)]
+        stream.synchronize()
+        # pass 1: back-to-back prepared calls, each bracketed by its own events
+        mon.set_state(blob, stream)
+        wall0 = time.time()
+        region[0].record(stream)
+        for j in range(K):
+            ev[j][0].record(stream)
+            calls[j]()
+            ev[j][1].record(stream)
+        region[1].record(stream)
+        stream.synchronize()
+        per_ms = [a.elapsed_time(b) for a, b in ev]
+        per_pass_counts.append(counts.cpu().numpy().copy())
+        rec["arenas"] = f"{K} distinct trace-step arenas, generated before timing"
+        rec["us_per_step"] = us(region[0].elapsed_time(region[1]) / K)
+        # pass 2: the K calls captured in one CUDA graph and replayed
+        mon.set_state(blob, stream)
+        graph = torch.cuda.CUDAGraph()
+        stream.synchronize()
+        with torch.cuda.graph(graph, stream=stream):
+            for j in range(K):
+                calls[j]()
+        graph.replay()                               # untimed: the first replay uploads the graph
+        mon.set_state(blob, stream)
+        torch.cuda.synchronize(dev)
+        region[0].record(stream)
+        graph.replay()
+        region[1].record(stream)
+        stream.synchronize()
+        g_ms = region[0].elapsed_time(region[1]) / K
+        per_pass_counts.append(counts.cpu().numpy().copy())
+        rec["graph_us_per_step"] = us(g_ms)
+        rec["graph_gbs"] = round(w.grad_bytes / (g_ms / 1e3) / 1e9, 1)
+        rec["graph_frac"] = round(w.grad_bytes / (g_ms / 1e3) / 1e9 / peak, 4)
+        del graph
+        # pass 3: L2 flushed (a 512 MB write) before every step, outside its events
+        if arena_bytes < 2e9:
+            flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+            mon.set_state(blob, stream)
+            for j in range(K):
+                flush.zero_()
+                ev[j][0].record(stream)
+                calls[j]()
+                ev[j][1].record(stream)
+            stream.synchronize()
+            fl = [a.elapsed_time(b) for a, b in ev]
+            per_pass_counts.append(counts.cpu().numpy().copy())
+            rec["l2_flushed_us_mean"] = us(statistics.mean(fl))
+            del flush
+        wall1 = time.time()
+        del calls, arenas
+    else:
+        ring = [scratch, filler.new_arena()]
+        clean = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+        clean_out = torch.empty((), dtype=torch.int64, device=dev)
+        wall0 = time.time()
+        for j in range(K):
+            a = ring[j % 2]
+            fill(a, t0 - 1 + j)
+            torch.sum(clean, dim=0, dtype=torch.int64, out=clean_out)
+            ev[j][0].record(stream)
+            mon.step(a, mask=mask, stats=step_stats[j], stream=stream)
+            ev[j][1].record(stream)
+        stream.synchronize()
+        wall1 = time.time()
+        per_ms = [a.elapsed_time(b) for a, b in ev]
+        per_pass_counts.append(counts.cpu().numpy().copy())
+        rec["arenas"] = ("two arenas, each regenerated with the next trace step between steps (outside the "
+                         "step's events), then a 512 MB read")
+        rec["us_per_step"] = us(statistics.mean(per_ms))
+        del ring, clean, clean_out
+    mon.close()
+    kern = statistics.mean(per_ms)
+    c = per_pass_counts[0]
+    rec.update({
+        "kernel_us_mean": us(kern), "kernel_us_min": us(min(per_ms)), "kernel_us_max": us(max(per_ms)),
+        "gbs": round(w.grad_bytes / (kern / 1e3) / 1e9, 1),
+        "frac": round(w.grad_bytes / (kern / 1e3) / 1e9 / peak, 4),
+        "candidates_mean": round(float(c[:, 0].mean()), 1), "candidates_max": int(c[:, 0].max()),
+        "selected_mean": round(float(c[:, 1].mean()), 2), "max_o": w.max_o,
+        "passes_agree": all(np.array_equal(c, x) for x in per_pass_counts[1:]),
+        "traffic": profiled_traffic(STEP_KERNEL_SOURCES, w.name),
+        "clocks": sampler.summary(wall0, wall1),
+    })
+    torch.cuda.synchronize(dev)
+    torch.cuda.empty_cache()
+    return rec
+
+
+def per_workload_records(args, dev, peak, peak_kind) -> dict:
+    """Every workload of --per-workload timed on its own trace steps (see
+    workload_record); frac is GB/s over the kernel mean against the peak."""
+    import torch
+    names = [n for n in args.per_workload.split(",") if n]
+    free, _ = torch.cuda.mem_get_info(dev)
+    budget = 0.45 * free
+    sampler = ClockSampler(dev.index)
+    time.sleep(0.3)
+    out = {"peak_gbs": peak, "peak_source": f"{peak_kind} hbm_gbs",
+           "what": ("per workload: trace steps t0..t0+K-1 of its own synthetic trace after a fresh monitor "
+                    "ran steps 1..t0-1; us_per_step = back-to-back prepared calls (distinct arenas) or the "
+                    "kernel mean (regenerated arenas); kernel_us_* from per-step CUDA events; gbs and frac "
+                    "from the kernel mean; candidates = |C_t| over the timed steps")}
+    try:
+        for n in names:
+            out[n] = workload_record(n, args.steps, args.warmup, dev, peak, sampler, budget)
+    finally:
+        sampler.stop()
+    return out
+
+
 def run_gnmr(args):
     import torch
     import workloads
@@ -388,6 +638,8 @@ def run_gnmr(args):
         with torch.cuda.graph(graph, stream=stream):
             for i in range(args.steps):
                 calls[(args.warmup + i) % n_arenas]()
+        with torch.cuda.stream(stream):
+            graph.replay()                # untimed: the first replay uploads the graph
         torch.cuda.synchronize(dev)
 
     sampler = ClockSampler(local_rank)
@@ -438,7 +690,7 @@ def run_gnmr(args):
     kern_ms = statistics.mean(per_ms)
     peak, peak_kind = measured_peaks()
     achieved = gbytes / (kern_ms / 1e3)
-    traffic = profiled_traffic(STEP_KERNEL_SOURCES)
+    traffic = profiled_traffic(STEP_KERNEL_SOURCES, w.name)
 
     # end to end through the public API with the step's input in pinned host
     # memory and its result read back to the host, every step inside the
@@ -515,12 +767,30 @@ def run_gnmr(args):
         cpu = {"value": round(rate, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
                "sample": (f"{what} ({int(w.lengths[units].sum()) * w.elem_bytes / 1e9:.3f} GB of "
                           f"{gbytes:.3f} GB per step): unit norms + Algorithms 1-2, "
-                          f"{sec:.2f} s wall on {threads} threads")}
+                          f"{sec:.2f} s wall on {threads} threads (contiguous unit groups of "
+                          f"equal bytes, each unit summed sequentially in double)")}
+        # one thread on a bounded prefix of the same layout (about 1.3 GB)
+        cum = np.cumsum(w.lengths[units]) * w.elem_bytes
+        one = units[:max(1, int(np.searchsorted(cum, 1.3e9)) + 1)]
+        rate1, _, sec1 = cpu_oracle_rate(view, w, one, threads=1)
+        cpu["single_thread"] = {
+            "value": round(rate1, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": (f"units 0..{len(one) - 1} of {w.num_units} "
+                       f"({int(w.lengths[one].sum()) * w.elem_bytes / 1e9:.3f} GB): unit norms + "
+                       f"Algorithms 1-2 on one thread, {sec1:.2f} s wall")}
     del host
 
     sparsity = None
     if rank == 0 and not args.no_sparsity:
         sparsity = trigger_sparsity(w, filler, arenas[0], dev)
+
+    per_workload = None
+    if rank == 0 and world == 1 and not args.no_per_workload and args.shrink == 1 and args.group == "tensor":
+        del calls, arenas, graph
+        mon.close()
+        torch.cuda.synchronize(dev)
+        torch.cuda.empty_cache()
+        per_workload = per_workload_records(args, dev, peak, peak_kind)
 
     if rank == 0:
         line = {
@@ -530,22 +800,15 @@ def run_gnmr(args):
             "pct_hbm_peak": round(100 * value / world / peak, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": w.dtype, "data": "synthetic",
-            "config": {"workload": f"{w.name} ({w.num_units} units, {w.num_segments} tensors, "
-                                   f"{w.grad_elems} {w.dtype} "
-                                   f"elements{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
-                       "bytes_per_step": w.grad_bytes, "arenas_cycled": n_arenas,
-                       "l2": ("L2 flushed before every step (512 MB write)" if args.flush_l2
-                              else "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * 129e6
-                              else "inputs fit in L2 (hot)"),
-                       "parallelism": "replicas" if world > 1 else "single GPU",
-                       "launch": ("one CUDA graph of the timed steps, replayed" if args.graph
-                                  else "one prepared gnmr_step call per step"),
+            "config": workload_config(w, args, n_arenas, world),
+            "launch": {"how": ("one CUDA graph of the timed steps, replayed" if args.graph
+                               else "one prepared gnmr_step call per step"),
                        "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
                                f"{info['num_warps']} warp runs, "
                                f"{'large-unit' if info['loop_shape'] == 2 else 'small-unit'} loop shape"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
-                         "traffic": traffic if w.name == "llama2-13b" and args.shrink == 1 else None,
+                         "traffic": traffic if args.shrink == 1 and args.group == "tensor" else None,
                          "traffic_unit": "bytes per launch (ncu dram__bytes_read+write)",
                          "algorithmic_bytes": w.grad_bytes,
                          "peak_source": f"{peak_kind} hbm_gbs", "kernel": f"gnmr_step_kernel<{w.dtype}>",
@@ -558,6 +821,8 @@ def run_gnmr(args):
             "clocks": clocks,
             "trigger_sparsity": sparsity,
         }
+        if per_workload is not None:
+            line["per_workload"] = per_workload
         print(json.dumps(line), flush=True)
     mon.close()
     if world > 1:

@@ -20,21 +20,29 @@ def test_traffic_record_follows_the_step_kernel_sources(tmp_path, monkeypatch):
         p.write_text(f"// source {i}\nint f{i}(int x) {{ return x + {i}; }}\n")
     prof = tmp_path / "profiles"
     prof.mkdir()
-    rec = {"kernel_source_sha256_16": bench.kernel_source_hash(srcs), "traffic_bytes_per_launch": 123}
+    rec = {"records": {"tiny": {"kernel_source_sha256_16": bench.kernel_source_hash(srcs),
+                                "traffic_bytes_per_launch": 123}}}
     (prof / "gnmr_step_kernel_traffic.json").write_text(json.dumps(rec))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.profiled_traffic(srcs) == 123
+    assert bench.profiled_traffic(srcs, "tiny") == 123
+    assert bench.profiled_traffic(srcs, "moe") is None          # no record for that workload
     srcs[1].write_text("/* reworded */ // source 1, still\nint f1(int x)  {  return x + 1; }\n")
-    assert bench.profiled_traffic(srcs) == 123        # comments and spacing only
+    assert bench.profiled_traffic(srcs, "tiny") == 123        # comments and spacing only
     srcs[1].write_text("// source 1\nint f1(int x) { return x + 2; }\n")
-    assert bench.profiled_traffic(srcs) is None
+    assert bench.profiled_traffic(srcs, "tiny") is None
 
 
-def test_committed_traffic_record_names_a_hash():
+def test_committed_traffic_records_name_a_hash():
+    import workloads
     with open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "profiles",
                            "gnmr_step_kernel_traffic.json")) as f:
-        rec = json.load(f)
-    assert len(rec["kernel_source_sha256_16"]) == 16 and rec["traffic_bytes_per_launch"] > 25_375_539_200
+        recs = json.load(f)["records"]
+    assert "llama2-13b" in recs
+    for name, rec in recs.items():
+        assert name in bench.PER_WORKLOADS
+        # every launch reads at least the gradient bytes once
+        assert len(rec["kernel_source_sha256_16"]) == 16
+        assert rec["traffic_bytes_per_launch"] >= workloads.make(name).grad_bytes
 
 
 def test_exceedance_counts_only_recoverable_units_strictly_over():
@@ -66,3 +74,46 @@ def test_reference_arm_prints_the_contract_line(capsys):
     e2e = line["e2e"]
     assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
+
+
+def test_trace_window_is_inside_the_trace_after_the_warmup():
+    for T, K, W in [(20, 20, 5), (50, 20, 5), (200, 20, 5), (100, 4, 3), (3, 10, 5), (50, 1, 0)]:
+        t0, k = bench.trace_window(T, K, W)
+        assert k >= 1 and t0 >= 1 and t0 + k - 1 == min(T, t0 + K - 1)
+        if T > W:
+            assert t0 >= W + 1 and k == min(K, T - W)
+    assert bench.trace_window(50, 20, 5) == (16, 20)          # centred: steps 16..35
+
+
+def test_host_arena_follows_the_layout_and_the_trace_scales():
+    """The reference arm's host-generated arena: the workload's packing,
+    zeros outside the units, every unit scaled by the power of two nearest
+    its trace scale (checked through the oracle's norms)."""
+    import numpy as np
+    import oracle
+    import workloads
+    w = workloads.make("tiny", shrink=8)
+    step = 7
+    units = np.arange(w.num_units)
+    a = bench.host_arena(w, step, units, 4)
+    assert a.dtype == np.float32 and a.size == w.arena_elems
+    inside = np.zeros(w.arena_elems, bool)
+    for o, n in zip(w.offsets, w.lengths):
+        inside[o:o + n] = True
+    assert np.all(a[~inside] == 0) and np.all(np.isfinite(a)) and np.all(a[inside] != 0)
+    # unit s holds block[start:start+n] * 2^k: its norm is 2^k times the block slice's
+    rng = np.random.default_rng([w.seed, 17, step])
+    block = rng.standard_normal(bench.HOST_BLOCK, dtype=np.float32)
+    block[np.abs(block) < 1e-6] = 1e-6
+    norms = oracle.unit_norms(a, w.offsets, w.lengths)
+    for s in (0, 5, w.num_units - 1):
+        k = int(round(np.log2(w.scales[step, s])))
+        start = (s * 7919) % bench.HOST_BLOCK
+        ref = oracle.unit_norms(block[start:start + w.lengths[s]], [0], [w.lengths[s]])[0]
+        assert norms[s] == ref * 2.0 ** k
+    b = workloads.make("llama2-13b", shrink=64)
+    h = bench.host_arena(b, 3, np.arange(b.num_units), 4)
+    assert h.dtype == np.uint16
+    bits = h[b.offsets[1]:b.offsets[1] + b.lengths[1]].astype(np.uint32) << 16
+    vals = bits.view(np.float32)
+    assert np.all(np.isfinite(vals)) and np.all(vals != 0)

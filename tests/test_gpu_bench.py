@@ -11,7 +11,8 @@ pytestmark = pytest.mark.gpu
 
 
 def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
-    bench.main(["--workload", "tiny", "--steps", "4", "--warmup", "3", "--e2e-steps", "3"])
+    bench.main(["--workload", "tiny", "--steps", "4", "--warmup", "3", "--e2e-steps", "3",
+                "--per-workload", "tiny,aq-stress"])
     line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
     assert line["metric"] == bench.METRIC and line["unit"] == "GB/s" and line["value"] > 0
     assert line["n_gpus"] == 1 and line["steps"] == 4 and line["warmup"] == 3
@@ -20,7 +21,7 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
     roof = line["roofline"]
     assert roof["bound"] == "hbm" and roof["unit"] == "GB/s" and roof["peak"] > 0
     assert roof["frac"] == pytest.approx(roof["achieved"] / roof["peak"], abs=1e-4)   # printed to 4 places
-    assert roof["traffic"] is None                     # recorded for the 13B layout only
+    assert roof["traffic"] is None or roof["traffic"] >= line["config"]["bytes_per_step"]
     cpu = line["cpu_baseline"]
     assert cpu["kind"] == "oracle" and cpu["value"] > 0 and cpu["cores"] >= 1 and cpu["sample"]
     e2e = line["e2e"]
@@ -32,3 +33,18 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(clocks)
     sparsity = line["trigger_sparsity"]
     assert sparsity["steps"] > 0 and 0 <= sparsity["selected_pct"] <= 100
+    assert cpu["single_thread"]["cores"] == 1 and cpu["single_thread"]["value"] > 0
+    per = line["per_workload"]
+    assert set(per) >= {"tiny", "aq-stress", "peak_gbs"}
+    for name, steps in (("tiny", 4), ("aq-stress", 4)):
+        rec = per[name]
+        assert rec["steps"] == steps and rec["trace_steps"][1] - rec["trace_steps"][0] + 1 == steps
+        assert rec["warmup_steps"] >= 3 and rec["passes_agree"] is True
+        for key in ("us_per_step", "kernel_us_mean", "kernel_us_min", "graph_us_per_step",
+                    "l2_flushed_us_mean"):
+            assert rec[key] > 0, key
+        assert rec["kernel_us_min"] <= rec["kernel_us_mean"] <= rec["kernel_us_max"]
+        assert rec["frac"] == pytest.approx(rec["gbs"] / per["peak_gbs"], abs=1e-3)
+        assert 0 <= rec["selected_mean"] <= rec["max_o"] and rec["candidates_max"] >= 0
+        assert {"sm_mhz", "reasons"} <= set(rec["clocks"])
+    assert per["aq-stress"]["candidates_mean"] > per["aq-stress"]["max_o"]   # the contended top-k
