@@ -306,6 +306,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         const size_t o_state = cv.take(sizeof(gnmr::UnitState) * U);
         const size_t o_queue = cv.take(sizeof(double) * U * c.window);
         const size_t o_cand = cv.take(sizeof(gnmr::Candidate) * U);
+        const uint32_t hot_cap = static_cast<uint32_t>(std::min<int64_t>(U, gnmr::kHotCapMax));
+        const size_t o_hot = cv.take(sizeof(gnmr::Candidate) * hot_cap);
+        const size_t o_hist = cv.take(sizeof(uint32_t) * gnmr::kRiskBins);
         const size_t o_ctl = cv.take(sizeof(gnmr::Control));
         const size_t o_cost = c.unit_cost ? cv.take(sizeof(double) * U) : 0;
 
@@ -326,6 +329,11 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         std::memcpy(&img[o_first], plan.first_warp.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_parts], plan.num_parts.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_pbase], plan.part_base.data(), sizeof(int64_t) * U);
+        {
+            gnmr::Control ctl{};
+            ctl.hot_bin = gnmr::kNoHot;              // no prediction before the first selection
+            std::memcpy(&img[o_ctl], &ctl, sizeof ctl);
+        }
 
         e = cudaMalloc(&h->dmem, cv.size);
         if (e != cudaSuccess) {
@@ -357,6 +365,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         p.state = reinterpret_cast<gnmr::UnitState *>(base + o_state);
         p.queue = reinterpret_cast<double *>(base + o_queue);
         p.cand = reinterpret_cast<gnmr::Candidate *>(base + o_cand);
+        p.hot = reinterpret_cast<gnmr::Candidate *>(base + o_hot);
+        p.hot_cap = hot_cap;
+        p.risk_hist = reinterpret_cast<uint32_t *>(base + o_hist);
         p.ctl = reinterpret_cast<gnmr::Control *>(base + o_ctl);
         p.unit_cost = c.unit_cost ? reinterpret_cast<const double *>(base + o_cost) : nullptr;
         p.policy = c.policy;
@@ -606,6 +617,7 @@ gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, i
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     gnmr::Control ctl{};
     ctl.steps = hdr.steps;
+    ctl.hot_bin = gnmr::kNoHot;
     cudaError_t e = cudaMemcpyAsync(h->params.state, in + sizeof hdr, units_bytes, cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(h->params.queue, in + sizeof hdr + units_bytes, queue_bytes,
@@ -614,6 +626,8 @@ gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, i
         e = cudaMemcpyAsync(h->params.ctl, &ctl, sizeof ctl, cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess)
         e = cudaMemsetAsync(h->params.unit_ticket, 0, sizeof(uint32_t) * h->num_units, st);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(h->params.risk_hist, 0, sizeof(uint32_t) * gnmr::kRiskBins, st);
     if (e == cudaSuccess)
         e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) {

@@ -52,11 +52,27 @@ struct Candidate {
 };
 constexpr uint32_t kCandActive = 0x80000000u;
 
+// Risk histogram of the candidate pool, built by the unit epilogues with one
+// atomic per pool member and read (and cleared) by the selecting CTA.  Bin 0
+// holds R < 1 (lock-only candidates); bin i >= 1 holds the R >= 1 whose
+// exponent and top three mantissa bits are the (i-1)-th such pattern above
+// 1.0: eight bins per octave, [1, 1.125), [1.125, 1.25), ..., [1.875, 2),
+// [2, 2.25), ...; the last bin also holds everything larger (+inf included).
+constexpr int kRiskBins = 2048;
+// Hot list: the candidates a step appends because their bin is at or above a
+// bin predicted from the previous step's cut (plus, under the admission cap,
+// every retained unit).  When the prediction holds, the selecting CTA reads
+// this short list instead of the whole candidate list.
+constexpr uint32_t kHotCapMax = 8192;
+constexpr uint32_t kNoHot = kRiskBins;   // hot_bin: no prediction, no pool member is hot
+
 // Device-resident step control block.
 struct Control {
     uint32_t ctas_done;   // CTA completion ticket of the current launch
     uint32_t n_cand;      // |C_t| appended so far
     int64_t steps;        // completed steps (t of the last step)
+    uint32_t n_hot;       // hot-list entries appended so far (may exceed the capacity)
+    uint32_t hot_bin;     // lowest bin whose pool members go to the hot list this step
 };
 
 // Checkpoint blob: this header, then UnitState[num_units], then the GNMR ring
@@ -86,6 +102,8 @@ struct StepParams {
     UnitState *state;            // [U]
     double *queue;               // [U * window] GNMR ring buffers
     Candidate *cand;             // [U]
+    Candidate *hot;              // [hot_cap] the hot list
+    uint32_t *risk_hist;         // [kRiskBins], zero between steps
     Control *ctl;
     uint8_t *mask;               // [U], caller
     double *out_norm, *out_gnmr, *out_dgnmr, *out_risk;  // caller, optional
@@ -99,7 +117,7 @@ struct StepParams {
     int64_t forced_steps;
     int64_t static_warmup;
     int32_t static_keep;                                  // ceil(static_fraction * |B_rec|)
-    int32_t pad2;
+    uint32_t hot_cap;                                     // min(U, kHotCapMax)
     int32_t num_units;
     int32_t num_warps;
     int32_t window;

@@ -80,6 +80,43 @@ __device__ __forceinline__ uint32_t index_key(int32_t b, int32_t num_units)
     return static_cast<uint32_t>(num_units - 1 - b);
 }
 
+// Bin of the risk histogram for a risk key (non-decreasing in the key): 0 for
+// R < 1, else 1 + the key's exponent and top three mantissa bits counted
+// from those of 1.0, the last bin open-ended.
+__device__ __forceinline__ uint32_t risk_bin(uint64_t key)
+{
+    constexpr uint32_t kOne = 1023u << 3;                 // exponent of 1.0, three mantissa bits 0
+    const uint32_t e8 = static_cast<uint32_t>(key >> 49); // sign (0), exponent, top three mantissa bits
+    if (e8 < kOne)
+        return 0;
+    const uint32_t b = e8 - kOne + 1;
+    return b < static_cast<uint32_t>(kRiskBins) ? b : static_cast<uint32_t>(kRiskBins - 1);
+}
+
+// Appends the lanes' entries (flag set) to a list with one atomic per warp;
+// slots at or past cap are counted but not written.  Called by all 32 lanes.
+__device__ __forceinline__ void warp_append(Candidate *list, uint32_t *count, uint32_t cap, bool flag, double r,
+                                            int32_t b, uint32_t lk)
+{
+    const unsigned want = __ballot_sync(kFull, flag);
+    if (!want)
+        return;
+    const int lane = threadIdx.x & 31;
+    const int leader = __ffs(want) - 1;
+    uint32_t base = 0;
+    if (lane == leader)
+        base = atomicAdd(count, static_cast<uint32_t>(__popc(want)));
+    base = __shfl_sync(kFull, base, leader);
+    if (flag) {
+        const uint32_t slot = base + __popc(want & ((1u << lane) - 1u));
+        if (slot < cap) {
+            list[slot].risk = r;
+            list[slot].unit = b;
+            list[slot].lock = lk;
+        }
+    }
+}
+
 // Unit epilogue for up to 32 units at once, one per lane (lanes with
 // `active` false only take part in the collective append): Algorithm 1, the
 // combined risk of Sec. 3.3, the statistics outputs and the candidate test of
@@ -191,23 +228,19 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
         }
         cand_lock = static_cast<uint32_t>(s.lock) | (s.active ? kCandActive : 0u);
     }
-    const unsigned want = __ballot_sync(kFull, cand);
-    if (want) {
-        const int lane = threadIdx.x & 31;
-        const int leader = __ffs(want) - 1;
-        uint32_t base = 0;
-        if (lane == leader)
-            base = atomicAdd(&p.ctl->n_cand, static_cast<uint32_t>(__popc(want)));
-        base = __shfl_sync(kFull, base, leader);
-        if (cand) {
-            const uint32_t slot = base + __popc(want & ((1u << lane) - 1u));
-            if (slot < static_cast<uint32_t>(p.num_units)) {   // at most one entry per unit
-                p.cand[slot].risk = r;
-                p.cand[slot].unit = b;
-                p.cand[slot].lock = cand_lock;
-            }
-        }
+    // The capped pool: every candidate, or under the admission cap those not
+    // active at t-1 (the retained ones are selected without ranking).  Pool
+    // members count in the risk histogram; the hot list takes those at or
+    // above this step's predicted bin, and every retained candidate.
+    const bool retained = cand && p.policy == 1 && (cand_lock & kCandActive);
+    bool hot = retained;
+    if (cand && !retained) {
+        const uint32_t bin = risk_bin(risk_key(r));
+        atomicAdd(&p.risk_hist[bin], 1u);
+        hot = bin >= __ldcg(&p.ctl->hot_bin);
     }
+    warp_append(p.cand, &p.ctl->n_cand, static_cast<uint32_t>(p.num_units), cand, r, b, cand_lock);
+    warp_append(p.hot, &p.ctl->n_hot, p.hot_cap, hot, r, b, cand_lock);
 }
 
 // A unit split over several warps: stores this warp's partial and takes a
@@ -350,19 +383,6 @@ __device__ void radix_select(const StepParams &p, uint32_t m, uint32_t K, bool o
     thr_lo = pre_lo;
 }
 
-// Block-wide sum of per-thread counts (all threads get it).
-__device__ __forceinline__ uint32_t block_count(uint32_t v, uint32_t *slot)
-{
-    if (threadIdx.x == 0)
-        *slot = 0;
-    __syncthreads();
-    v = __reduce_add_sync(kFull, v);
-    if ((threadIdx.x & 31) == 0 && v)
-        atomicAdd(slot, v);
-    __syncthreads();
-    return *slot;
-}
-
 // Delta M_t = sum of c_b over the units on the recovery path, in a fixed
 // order (thread-strided partial sums, then a fixed tree), so the value is
 // reproducible run to run.
@@ -398,32 +418,34 @@ __device__ __forceinline__ void commit_selected(const StepParams &p, bool stat, 
     }
 }
 
-// The selecting CTA's copy of the candidates' risk keys: candidate i's
-// risk_key in keys[i] and whether it belongs to the capped pool in bit i of
-// pool_bits (the candidates outside it -- retained under the admission cap --
-// are selected without ranking), followed by the radix histogram.  One read
-// of the candidate list fills it; the radix passes then run on shared memory
-// with 11-bit digits (2048 bins), so a 64-bit key needs at most six passes
-// and risks that crowd into one octave usually resolve in three.
+// The selecting CTA's shared memory: the cut list (the pool members of the
+// bin that holds the maxO-th largest risk, when only part of that bin is
+// selected: key, unit, lock word) and, for a cut bin too large to rank
+// directly, the histogram of an in-CTA radix select over it.
 constexpr int kWideBits = 11;
 constexpr int kWideBins = 1 << kWideBits;
 static_assert(kWideBins == 4 * kThreads, "four histogram bins per thread of the selecting CTA");
-constexpr uint32_t kKeyCache = 6144;
-constexpr size_t kKeyBitsOffset = sizeof(uint64_t) * kKeyCache;
-constexpr size_t kKeyHistOffset = kKeyBitsOffset + sizeof(uint32_t) * (kKeyCache / 32);
-constexpr size_t kKeyCacheBytes = kKeyHistOffset + sizeof(uint32_t) * kWideBins;
-static_assert(kKeyHistOffset % 16 == 0, "the histogram is read as 16-byte vectors");
+static_assert(kRiskBins == 4 * kThreads, "four risk-histogram bins per thread of the selecting CTA");
+constexpr uint32_t kCutCap = 3072;
+constexpr size_t kCutUnitOffset = sizeof(uint64_t) * kCutCap;
+constexpr size_t kCutLockOffset = kCutUnitOffset + sizeof(int32_t) * kCutCap;
+constexpr size_t kCutHistOffset = kCutLockOffset + sizeof(uint32_t) * kCutCap;
+constexpr size_t kKeyCacheBytes = kCutHistOffset + sizeof(uint32_t) * kWideBins;
+static_assert(kCutHistOffset % 16 == 0, "the histogram is read as 16-byte vectors");
 
-__device__ __forceinline__ bool in_pool(const uint32_t *pool_bits, uint32_t i)
-{
-    return (pool_bits[i >> 5] >> (i & 31u)) & 1u;
-}
+// Slots of the selecting CTA's misc[] words.
+constexpr int kMiscLast = 0;      // this CTA took the last grid ticket
+constexpr int kMiscBin = 1;       // find_*: the bin holding the r-th largest
+constexpr int kMiscRank = 2;      // r minus the count above that bin
+constexpr int kMiscCount = 3;     // that bin's count
+constexpr int kMiscHint = 5;      // scan_risk_hist: the bin holding the hint-th largest
+constexpr int kMiscPool = 6;      // scan_risk_hist: the pool size
+constexpr int kMiscFill = 7;      // cut-list entries appended
 
-// Bucket of the r-th largest digit in hist[kWideBins] (r >= 1), by the whole
+// Bin of the r-th largest digit in hist[kWideBins] (r >= 1), by the whole
 // CTA: thread t owns the four bins just below those of thread t - 1 (thread
 // 0 the highest); the counts above each thread's bins come from a warp scan
-// and a scan of the 16 warp totals (in wsum[16]).  misc[1] = the bucket,
-// misc[2] = r minus the count above it, misc[3] = its count.
+// and a scan of the 16 warp totals (in wsum[16]).
 __device__ __forceinline__ void find_bucket_wide(const uint32_t *hist, uint32_t r, uint32_t *misc, uint32_t *wsum)
 {
     const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
@@ -459,9 +481,9 @@ __device__ __forceinline__ void find_bucket_wide(const uint32_t *hist, uint32_t 
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             if (above + c4[j] >= r) {
-                misc[1] = static_cast<uint32_t>(4 * q4 + 3 - j);
-                misc[2] = r - above;
-                misc[3] = c4[j];
+                misc[kMiscBin] = static_cast<uint32_t>(4 * q4 + 3 - j);
+                misc[kMiscRank] = r - above;
+                misc[kMiscCount] = c4[j];
                 break;
             }
             above += c4[j];
@@ -469,23 +491,133 @@ __device__ __forceinline__ void find_bucket_wide(const uint32_t *hist, uint32_t 
     }
 }
 
-// K-th largest (risk_key : index_key) among the pool's m <= kKeyCache cached
-// keys, 1 <= K < pool size: MSD radix select with 11-bit digits over the
-// cached 64-bit keys, then, only if whole keys tie at the cut, over the unit
-// indices (read from the candidate list).  Exactly K pool keys compare >= the
-// returned threshold.  whole_pool: every cached candidate belongs to the
-// pool (no admission cap), so pool_bits is not read.  All threads of the CTA
-// call this.
-__device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K, const uint64_t *keys,
-                                    const uint32_t *pool_bits, bool whole_pool, uint32_t *hist, uint32_t *wsum,
-                                    uint32_t *misc, uint64_t &thr_hi, uint32_t &thr_lo)
+// Reads and clears the global risk histogram (four bins per thread, thread 0
+// the highest).  misc[kMiscPool] = the pool size P; with K = min(P, cap),
+// if 1 <= K < P: misc[kMiscBin/Rank/Count] describe the bin holding the K-th
+// largest risk, and misc[kMiscHint] the bin holding the min(P, K + extra)-th
+// largest (the next step's hot-list prediction).  Callers synchronise after.
+__device__ void scan_risk_hist(const StepParams &p, uint32_t cap, uint32_t extra, uint32_t *misc, uint32_t *wsum)
 {
-    const int lo_bits = p.num_units > 1 ? 32 - __clz(static_cast<uint32_t>(p.num_units - 1)) : 0;
-    const uint32_t lane = threadIdx.x & 31u;
-    uint64_t pre_hi = 0, msk_hi = 0;
+    const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
+    const int q4 = kRiskBins / 4 - 1 - t;
+    uint4 *gh = reinterpret_cast<uint4 *>(p.risk_hist) + q4;
+    const uint4 q = __ldcg(gh);                                      // bins 4 q4 .. 4 q4 + 3
+    __stcg(gh, make_uint4(0u, 0u, 0u, 0u));                          // empty for the next step
+    const uint32_t c4[4] = {q.w, q.z, q.y, q.x};                     // descending
+    const uint32_t sum = c4[0] + c4[1] + c4[2] + c4[3];
+    uint32_t incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t u = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o)
+            incl += u;
+    }
+    if (lane == 31)
+        wsum[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+        const uint32_t tot = lane < kWarpsPerCta ? wsum[lane] : 0u;
+        uint32_t x = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t u = __shfl_up_sync(kFull, x, o);
+            if (lane >= o)
+                x += u;
+        }
+        if (lane < kWarpsPerCta)
+            wsum[lane] = x - tot;
+        if (lane == kWarpsPerCta - 1)
+            misc[kMiscPool] = x;
+    }
+    __syncthreads();
+    const uint32_t pool = misc[kMiscPool];
+    const uint32_t K = pool < cap ? pool : cap;
+    if (K == 0 || K >= pool)
+        return;
+    const uint32_t r2 = pool - K > extra ? K + extra : pool;
+    const uint32_t above0 = wsum[wid] + incl - sum;
+    if (above0 < K && K <= above0 + sum) {
+        uint32_t above = above0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (above + c4[j] >= K) {
+                misc[kMiscBin] = static_cast<uint32_t>(4 * q4 + 3 - j);
+                misc[kMiscRank] = K - above;
+                misc[kMiscCount] = c4[j];
+                break;
+            }
+            above += c4[j];
+        }
+    }
+    if (above0 < r2 && r2 <= above0 + sum) {
+        uint32_t above = above0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (above + c4[j] >= r2) {
+                misc[kMiscHint] = static_cast<uint32_t>(4 * q4 + 3 - j);
+                break;
+            }
+            above += c4[j];
+        }
+    }
+}
+
+// One read of n list entries: commits every retained entry (admission cap)
+// and every pool entry in a bin above c; the pool entries of bin c are
+// committed too when the whole bin is selected, else collected in the cut
+// list (misc[kMiscFill] counts them; at most kCutCap are stored).
+__device__ void gather_commit(const StepParams &p, const Candidate *src, uint32_t n, bool admission, bool stat,
+                              uint32_t c, bool whole_bin, uint64_t *ck, int32_t *cu, uint32_t *cl, uint32_t *misc)
+{
+    for (uint32_t i0 = threadIdx.x; i0 < n; i0 += kSelectIlp * blockDim.x) {
+        double rr[kSelectIlp];
+        int32_t bb[kSelectIlp];
+        uint32_t ll[kSelectIlp];
+#pragma unroll
+        for (int j = 0; j < kSelectIlp; ++j) {      // loads in flight per thread
+            const uint32_t i = i0 + j * blockDim.x;
+            if (i < n)
+                load_candidate(src + i, rr[j], bb[j], ll[j]);
+        }
+#pragma unroll
+        for (int j = 0; j < kSelectIlp; ++j) {
+            if (i0 + j * blockDim.x >= n)
+                break;
+            if (admission && (ll[j] & kCandActive)) {
+                commit_selected(p, stat, bb[j], rr[j], ll[j]);
+                continue;
+            }
+            const uint64_t key = risk_key(rr[j]);
+            const uint32_t bin = risk_bin(key);
+            if (bin > c || (bin == c && whole_bin)) {
+                commit_selected(p, stat, bb[j], rr[j], ll[j]);
+            } else if (bin == c) {
+                const uint32_t at = atomicAdd(&misc[kMiscFill], 1u);
+                if (at < kCutCap) {
+                    ck[at] = key;
+                    cu[at] = bb[j];
+                    cl[at] = ll[j];
+                }
+            }
+        }
+    }
+}
+
+// r-th largest (key : index_key) among the n <= kCutCap cut-list entries,
+// 1 <= r < n: MSD radix select with 11-bit digits on shared memory, starting
+// at bit `start` of the 64-bit key (the bits above it are equal for every
+// entry), then over the unit indices when whole keys tie.  Exactly r entries
+// compare >= the returned threshold.  All threads of the CTA call this.
+__device__ void radix_select_cut(const uint64_t *keys, const int32_t *units, uint32_t n, uint32_t r, int start,
+                                 int32_t num_units, uint32_t *hist, uint32_t *wsum, uint32_t *misc,
+                                 uint64_t &thr_hi, uint32_t &thr_lo)
+{
+    const int lo_bits = num_units > 1 ? 32 - __clz(static_cast<uint32_t>(num_units - 1)) : 0;
+    uint64_t pre_hi = 0, msk_hi = start < 64 ? ~0ull << start : 0ull;
+    if (start < 64)
+        pre_hi = keys[0] & msk_hi;
     uint32_t pre_lo = 0, msk_lo = 0;
-    uint32_t r = K;
-    int pos_hi = 64, pos_lo = lo_bits;               // bits of each key part not yet decided
+    int pos_hi = start, pos_lo = lo_bits;
     while (pos_hi > 0 || pos_lo > 0) {
         const bool in_hi = pos_hi > 0;
         int &pos = in_hi ? pos_hi : pos_lo;
@@ -495,38 +627,27 @@ __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K,
         const uint32_t dmask = (1u << width) - 1u;
         reinterpret_cast<uint4 *>(hist)[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
         __syncthreads();
-        // four keys per thread per iteration (independent chains)
-        for (uint32_t w0 = threadIdx.x & ~31u; w0 < m; w0 += 4 * blockDim.x) {
-            bool take[4];
-            uint32_t dig[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const uint32_t i = w0 + j * blockDim.x + lane;
-                take[j] = i < m && (whole_pool || in_pool(pool_bits, i));
-                dig[j] = 0;
-                if (take[j]) {
-                    const uint64_t hi = keys[i];
-                    take[j] = (hi & msk_hi) == pre_hi;
-                    if (in_hi) {
-                        dig[j] = static_cast<uint32_t>(hi >> shift) & dmask;
-                    } else if (take[j]) {           // whole keys tie: rank by unit index
-                        const uint32_t lo = index_key(__ldcg(&p.cand[i].unit), p.num_units);
-                        take[j] = (lo & msk_lo) == pre_lo;
-                        dig[j] = (lo >> shift) & dmask;
-                    }
-                }
+        for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
+            const uint64_t hi = keys[i];
+            if ((hi & msk_hi) != pre_hi)
+                continue;
+            uint32_t dig;
+            if (in_hi) {
+                dig = static_cast<uint32_t>(hi >> shift) & dmask;
+            } else {                                  // whole keys tie: rank by unit index
+                const uint32_t lo = index_key(units[i], num_units);
+                if ((lo & msk_lo) != pre_lo)
+                    continue;
+                dig = (lo >> shift) & dmask;
             }
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-                if (take[j])
-                    atomicAdd(&hist[dig[j]], 1u);
+            atomicAdd(&hist[dig], 1u);
         }
         __syncthreads();
         find_bucket_wide(hist, r, misc, wsum);
         __syncthreads();
-        const uint32_t bucket = misc[1];
-        const uint32_t in_bucket = misc[3];
-        r = misc[2];
+        const uint32_t bucket = misc[kMiscBin];
+        const uint32_t in_bucket = misc[kMiscCount];
+        r = misc[kMiscRank];
         if (in_hi) {
             pre_hi |= static_cast<uint64_t>(bucket) << shift;
             msk_hi |= static_cast<uint64_t>(dmask) << shift;
@@ -542,11 +663,51 @@ __device__ void radix_select_cached(const StepParams &p, uint32_t m, uint32_t K,
     thr_lo = pre_lo;
 }
 
+// Commits the r largest (key desc, unit asc) of the n cut-list entries,
+// 1 <= r < n <= kCutCap.  Up to one entry per thread: each entry's rank is
+// counted against all others directly; larger lists use the radix select.
+__device__ void select_cut(const StepParams &p, bool stat, uint32_t c, uint32_t n, uint32_t r, const uint64_t *ck,
+                           const int32_t *cu, const uint32_t *cl, uint32_t *hist, uint32_t *wsum, uint32_t *misc)
+{
+    if (n <= blockDim.x) {
+        const uint32_t i = threadIdx.x;
+        if (i < n) {
+            const uint64_t k = ck[i];
+            const int32_t u = cu[i];
+            uint32_t rank = 0;
+            for (uint32_t j = 0; j < n; ++j) {
+                const uint64_t kj = ck[j];
+                rank += (kj > k || (kj == k && cu[j] < u)) ? 1u : 0u;
+            }
+            if (rank < r)
+                commit_selected(p, stat, u, __longlong_as_double(static_cast<long long>(k)), cl[i]);
+        }
+        return;
+    }
+    // every key of an interior bin shares the sign, exponent and top three mantissa bits
+    const int start = (c > 0 && c + 1 < static_cast<uint32_t>(kRiskBins)) ? 49 : 64;
+    uint64_t thr_hi = 0;
+    uint32_t thr_lo = 0;
+    radix_select_cut(ck, cu, n, r, start, p.num_units, hist, wsum, misc, thr_hi, thr_lo);
+    for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
+        const uint64_t k = ck[i];
+        if (k > thr_hi || (k == thr_hi && index_key(cu[i], p.num_units) >= thr_lo))
+            commit_selected(p, stat, cu[i], __longlong_as_double(static_cast<long long>(k)), cl[i]);
+    }
+}
+
 // Last CTA: Top_maxO (or the policy's choice), Algorithm 2's lock
 // bookkeeping, mask, counts, Delta M_t, reset.  The unit epilogues have
 // already written the outcome of every unit outside A_t; this writes A_t.
+//
+// The risk histogram gives the pool size and the bin c that holds the
+// maxO-th largest risk.  One read of a list then commits every entry above c
+// (and the retained ones), and the pool members of bin c are ranked among
+// themselves.  The list read is the hot list when the previous step's
+// prediction was at or below c and the hot list did not overflow (it then
+// holds every entry at or above c), else the whole candidate list.
 __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist, uint32_t *misc, double *red,
-                                  unsigned char *key_cache)
+                                  unsigned char *smem)
 {
     uint32_t m = __ldcg(&p.ctl->n_cand);
     m = m < static_cast<uint32_t>(p.num_units) ? m : static_cast<uint32_t>(p.num_units);
@@ -554,6 +715,7 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
     const bool stat = p.policy == 2 && !all_on;
     const bool admission = p.policy == 1 && !all_on;
     uint32_t n_sel = 0;
+    uint32_t next_hot = kNoHot + 1;                  // > kNoHot: keep the current prediction
     if (all_on) {
         m = 0;
         n_sel = static_cast<uint32_t>(p.num_recoverable);
@@ -561,20 +723,15 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
         m = 0;
         n_sel = static_cast<uint32_t>(p.static_keep);
     } else {
-        // the pool the cap applies to: every candidate, or the new ones only
-        uint32_t pool = m;
-        uint32_t retained = 0;
-        if (admission) {
-            uint32_t mine = 0;
-            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x)
-                mine += (__ldcg(&p.cand[i].lock) & kCandActive) ? 1u : 0u;
-            retained = block_count(mine, &misc[4]);     // misc[0] holds the last-CTA flag
-            pool = m - retained;
-        }
         const uint32_t cap = stat ? static_cast<uint32_t>(p.static_keep) : static_cast<uint32_t>(p.max_o);
+        scan_risk_hist(p, cap, 3 * cap + 64, misc, hist);
+        __syncthreads();
+        const uint32_t pool = misc[kMiscPool];
+        const uint32_t retained = admission && m > pool ? m - pool : 0u;
         const uint32_t K = pool < cap ? pool : cap;
-        const bool take_all = pool <= cap;
-        if (take_all || K == 0) {
+        if (K == 0 || K >= pool) {
+            // the whole pool is selected (or none of it): one read of the list
+            const bool take_all = K >= pool;
             for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
                 double r;
                 int32_t b;
@@ -583,69 +740,44 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
                 if (take_all || (admission && (lk & kCandActive)))
                     commit_selected(p, stat, b, r, lk);
             }
-        } else if (m <= kKeyCache) {
-            uint64_t *keys = reinterpret_cast<uint64_t *>(key_cache);
-            uint32_t *pool_bits = reinterpret_cast<uint32_t *>(key_cache + kKeyBitsOffset);
-            uint32_t *wide_hist = reinterpret_cast<uint32_t *>(key_cache + kKeyHistOffset);
-            const uint32_t lane = threadIdx.x & 31u;
-            // one read of the candidate list (loads in flight per thread)
-            for (uint32_t w0 = (threadIdx.x & ~31u); w0 < m; w0 += kSelectIlp * blockDim.x) {
-                double rr[kSelectIlp];
-                uint32_t ll[kSelectIlp];
-#pragma unroll
-                for (int j = 0; j < kSelectIlp; ++j) {
-                    const uint32_t i = w0 + j * blockDim.x + lane;
-                    int32_t b;
-                    if (i < m)
-                        load_candidate(p.cand + i, rr[j], b, ll[j]);
-                }
-#pragma unroll
-                for (int j = 0; j < kSelectIlp; ++j) {
-                    const uint32_t i = w0 + j * blockDim.x + lane;
-                    const bool member = i < m && !(admission && (ll[j] & kCandActive));
-                    const unsigned word = __ballot_sync(kFull, member);
-                    if (i < m)
-                        keys[i] = risk_key(rr[j]);
-                    if (lane == 0 && w0 + j * blockDim.x < m)
-                        pool_bits[(w0 + j * blockDim.x) >> 5] = word;
-                }
-            }
-            __syncthreads();
-            uint64_t thr_hi = 0;
-            uint32_t thr_lo = 0;
-            radix_select_cached(p, m, K, keys, pool_bits, !admission, wide_hist, hist, misc, thr_hi, thr_lo);
-            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
-                bool sel;
-                if (admission && !in_pool(pool_bits, i)) {
-                    sel = true;                              // retained outside the cap
-                } else {
-                    const uint64_t key = keys[i];
-                    sel = key > thr_hi ||
-                          (key == thr_hi && index_key(__ldcg(&p.cand[i].unit), p.num_units) >= thr_lo);
-                }
-                if (sel) {
-                    double r;
-                    int32_t b;
-                    uint32_t lk;
-                    load_candidate(p.cand + i, r, b, lk);
-                    commit_selected(p, stat, b, r, lk);
-                }
-            }
+            next_hot = 0;                            // a small pool: every candidate is hot next step
         } else {
-            // more candidates than the shared-memory cache: radix passes over
-            // the candidate list in global memory
-            uint64_t thr_hi = 0;
-            uint32_t thr_lo = 0;
-            radix_select(p, m, K, admission, hist, misc, thr_hi, thr_lo);
-            for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
-                double r;
-                int32_t b;
-                uint32_t lk;
-                load_candidate(p.cand + i, r, b, lk);
-                const uint64_t key = risk_key(r);
-                if ((admission && (lk & kCandActive)) || key > thr_hi ||
-                    (key == thr_hi && index_key(b, p.num_units) >= thr_lo))
-                    commit_selected(p, stat, b, r, lk);
+            uint64_t *ck = reinterpret_cast<uint64_t *>(smem);
+            int32_t *cu = reinterpret_cast<int32_t *>(smem + kCutUnitOffset);
+            uint32_t *cl = reinterpret_cast<uint32_t *>(smem + kCutLockOffset);
+            uint32_t *wide_hist = reinterpret_cast<uint32_t *>(smem + kCutHistOffset);
+            const uint32_t c = misc[kMiscBin], rc = misc[kMiscRank], nc = misc[kMiscCount];
+            next_hot = misc[kMiscHint];
+            const uint32_t hot_bin = __ldcg(&p.ctl->hot_bin);
+            const uint32_t n_hot = __ldcg(&p.ctl->n_hot);
+            const bool use_hot = hot_bin <= c && n_hot <= p.hot_cap;
+            __syncthreads();                         // every thread has read misc
+            if (threadIdx.x == 0)
+                misc[kMiscFill] = 0;
+            __syncthreads();
+            gather_commit(p, use_hot ? p.hot : p.cand, use_hot ? n_hot : m, admission, stat, c, rc == nc,
+                          ck, cu, cl, misc);
+            __syncthreads();
+            if (rc < nc) {
+                if (nc <= kCutCap) {
+                    select_cut(p, stat, c, nc, rc, ck, cu, cl, wide_hist, hist, misc);
+                } else {
+                    // a cut bin larger than the shared list: radix passes over the
+                    // whole candidate list in global memory (commits are idempotent)
+                    uint64_t thr_hi = 0;
+                    uint32_t thr_lo = 0;
+                    radix_select(p, m, K, admission, hist, misc, thr_hi, thr_lo);
+                    for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+                        double r;
+                        int32_t b;
+                        uint32_t lk;
+                        load_candidate(p.cand + i, r, b, lk);
+                        const uint64_t key = risk_key(r);
+                        if ((admission && (lk & kCandActive)) || key > thr_hi ||
+                            (key == thr_hi && index_key(b, p.num_units) >= thr_lo))
+                            commit_selected(p, stat, b, r, lk);
+                    }
+                }
             }
         }
         n_sel = K + retained;
@@ -662,6 +794,9 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
     __syncthreads();
     if (threadIdx.x == 0) {
         p.ctl->n_cand = 0;
+        p.ctl->n_hot = 0;
+        if (next_hot <= kNoHot)
+            p.ctl->hot_bin = next_hot;
         p.ctl->ctas_done = 0;
         p.ctl->steps += 1;
     }

@@ -8,11 +8,15 @@ same n_b (the oracle gets sqrt of the same sums of squares) and run the same
 correctly rounded fp64 operations, so R, the masks, the locks and the counts
 must agree exactly -- no decision margin is needed, and ties are real.
 
-The cases steer the selection through each of its paths: the cut bucket of
-the coarse risk histogram ranked in shared memory, a cut bucket taken whole,
-a cut bucket at and just past the shared list's capacity (the exact radix
-select), equal risks inside the cut bucket, lock-only candidates, and the
-admission-cap and static policies."""
+The cases steer the selection through each of its paths.  The risk
+histogram (eight bins per octave: exponent and top three mantissa bits)
+locates the cut bin; its members are ranked directly (up to 512), by a radix
+select in shared memory (up to 3,072), or by radix passes over the whole
+candidate list in global memory (more); a cut bin can also be taken whole.
+Multi-step cases drive the hot list: the previous step's prediction held
+(only the hot list is read), missed (the risks fell below it), or the hot
+list overflowed.  Equal risks inside the cut bin, lock-only candidates and
+the admission-cap and static policies are covered too."""
 import numpy as np
 import pytest
 
@@ -56,10 +60,14 @@ def _whole_bucket(rng):
 CASES = {
     "spread": _spread,
     "narrow_overflow": _narrow,
-    "cut_500": _with_cut_members(500),
-    "cut_at_capacity": _with_cut_members(1014),
-    "cut_past_capacity": _with_cut_members(1100),
+    "cut_55": _with_cut_members(55),
+    "cut_512": _with_cut_members(512),
+    "cut_513": _with_cut_members(513),
+    "cut_1500": _with_cut_members(1500),
+    "cut_at_capacity": _with_cut_members(3072),
+    "cut_past_capacity": _with_cut_members(3073),
     "cut_ties": _with_cut_members(300, ties=True),
+    "cut_ties_radix": _with_cut_members(2000, ties=True),
     "whole_bucket": _whole_bucket,
 }
 
@@ -100,6 +108,33 @@ def test_top_max_o_paths(case, cuda_device):
     rng = np.random.default_rng(sorted(CASES).index(case) + 101)
     res = _drive([CASES[case](rng)])
     assert res.n_selected == MAX_O
+
+
+def _scaled(factor):
+    def make(rng):
+        return _spread(rng) * factor
+    return make
+
+
+HOT_SEQUENCES = {
+    # the same distribution every step: from step 3 on the prediction holds
+    "stationary": [_spread] * 5,
+    # risks shift down by 100x: the cut falls below the predicted bin (full list)
+    "shift_down": [_spread, _spread, _scaled(0.01), _scaled(0.01), _spread],
+    # risks shift up by 100x: the cut rises above the prediction (hot list holds more)
+    "shift_up": [_spread, _spread, _scaled(100.0), _spread],
+    # a step whose pool fits the budget (every candidate hot next step), then a
+    # step with ~20,000 candidates: the hot list overflows (full list)
+    "overflow": [lambda rng: np.full(U, 0.5), _with_cut_members(20, ties=False), _narrow, _spread],
+    # a cut bin ranked by the shared-memory radix select out of the hot list
+    "hot_radix": [_with_cut_members(1500), _with_cut_members(1500), _with_cut_members(1500)],
+}
+
+
+@pytest.mark.parametrize("seq", sorted(HOT_SEQUENCES))
+def test_hot_list_predictions(seq, cuda_device):
+    rng = np.random.default_rng(sorted(HOT_SEQUENCES).index(seq) + 301)
+    _drive([make(rng) for make in HOT_SEQUENCES[seq]])
 
 
 def test_lock_only_candidates_compete_with_new_spikes(cuda_device):
