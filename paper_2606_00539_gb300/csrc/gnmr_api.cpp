@@ -329,6 +329,8 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         std::memcpy(&img[o_first], plan.first_warp.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_parts], plan.num_parts.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_pbase], plan.part_base.data(), sizeof(int64_t) * U);
+        std::memset(&img[o_partial], 0xff, sizeof(double) * plan.num_partials);   // every slot empty
+        static_assert(gnmr::kEmptyPartial == ~0ull, "empty partial slots are all-ones bytes");
         {
             gnmr::Control ctl{};
             ctl.hot_bin = gnmr::kNoHot;              // no prediction before the first selection
@@ -628,6 +630,8 @@ gnmr_status gnmr_set_state(gnmr_handle *h, void *stream, const void *host_buf, i
         e = cudaMemsetAsync(h->params.unit_ticket, 0, sizeof(uint32_t) * h->num_units, st);
     if (e == cudaSuccess)
         e = cudaMemsetAsync(h->params.risk_hist, 0, sizeof(uint32_t) * gnmr::kRiskBins, st);
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(h->params.partial, 0xff, sizeof(double) * h->num_partials, st);
     if (e == cudaSuccess)
         e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) {

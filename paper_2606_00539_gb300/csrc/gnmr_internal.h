@@ -43,6 +43,11 @@ struct UnitState {
 static_assert(offsetof(UnitState, lock) % 8 == 0 && offsetof(UnitState, active) == offsetof(UnitState, lock) + 4,
               "UnitState lock/active pair");
 
+// Bit pattern of an empty partial slot (a NaN that no partial sum takes:
+// partials are non-negative, +inf or the canonical NaN).  The first slot of
+// every unit split in two holds it between steps.
+constexpr unsigned long long kEmptyPartial = ~0ull;
+
 // Candidate-pool entry written by the unit epilogue, read by the selection
 // (one 16-byte load).
 struct Candidate {

@@ -245,11 +245,30 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
 
 // A unit split over several warps: stores this warp's partial and takes a
 // ticket.  Returns true (with the unit's total in s) for the warp that takes
-// the last ticket; that warp sums the partials in slot order.
+// the last ticket; that warp sums the partials in slot order.  A unit of two
+// parts trades its partial through the first slot in one atomic exchange:
+// the first warp finds the slot empty and leaves its partial there, the
+// second takes it, adds it to its own (IEEE addition is commutative, so the
+// bits are those of the slot-order sum) and empties the slot again.
 __device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, int32_t parts, int warp,
                                               double &s, int lane)
 {
     const int64_t base = p.part_base[b];
+    if (parts == 2) {
+        unsigned long long other = 0;
+        if (lane == 0) {
+            const double mine = isnan(s) ? CUDART_NAN : s;          // never the empty pattern
+            other = atomicExch(reinterpret_cast<unsigned long long *>(p.partial + base),
+                               static_cast<unsigned long long>(__double_as_longlong(mine)));
+        }
+        other = __shfl_sync(kFull, other, 0);
+        if (other == kEmptyPartial)
+            return false;
+        if (lane == 0)
+            __stcg(reinterpret_cast<unsigned long long *>(p.partial + base), kEmptyPartial);
+        s = s + __longlong_as_double(static_cast<long long>(other));
+        return true;
+    }
     uint32_t last = 0;
     if (lane == 0) {
         __stcg(&p.partial[base + (warp - p.first_warp[b])], s);
@@ -916,9 +935,9 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     // every CTA's writes.
     __syncthreads();
     if (threadIdx.x == 0)
-        s_misc[0] = ticket_acq_rel(&p.ctl->ctas_done) == gridDim.x - 1 ? 1u : 0u;
+        s_misc[kMiscLast] = ticket_acq_rel(&p.ctl->ctas_done) == gridDim.x - 1 ? 1u : 0u;
     __syncthreads();
-    if (s_misc[0]) {
+    if (s_misc[kMiscLast]) {
         select_and_commit(p, __ldcg(&p.ctl->steps) + 1, s_hist, s_misc, s_red, s_keys);
     }
 }
