@@ -31,7 +31,8 @@
  *     rescale.  The paper fixes no precision for this arithmetic; the reading
  *     taken is fp32 throughout (inv = fmax / amax, v = x * inv, y = q * (amax /
  *     fmax)), ties to the even code, saturation at fmax, rows whose max is 0
- *     or that hold a NaN or Inf left unchanged.
+ *     or that hold a NaN or Inf left unchanged, and so are rows whose scale
+ *     factor fmax / amax overflows fp32 (amax below fmax / FLT_MAX).
  *
  * Build: gcc -O2 -std=c11 -ffp-contract=off -shared -fPIC -o liboracle_gnmr.so
  * gnmr_oracle.c -lm (no fast-math, no fused multiply-add: every operation
@@ -551,6 +552,8 @@ int oracle_fake_quant(const void *in, void *out, int dtype, int64_t rows, int64_
                 amax = fabsf(x);
         }
         int keep = code == 0 || amax == 0.0f || nonfinite;
+        if (!keep && isinf(f.fmax / amax))
+            keep = 1;   /* the row's scale factor overflows fp32: left unchanged, like a zero row */
         float inv = keep ? 1.0f : f.fmax / amax;
         float scale = keep ? 1.0f : amax / f.fmax;
         for (int64_t c = 0; c < cols; ++c) {

@@ -5,7 +5,8 @@
 // y = round_to_format(x * inv) * scale, rounding to the nearest representable
 // value with ties to the even code and saturating at fmax.  All arithmetic is
 // fp32, so the quantized codes are the same on any IEEE machine.  Rows whose
-// max is 0, or that hold a NaN or Inf, are copied unchanged.
+// max is 0, that hold a NaN or Inf, or whose scale factor fmax / amax
+// overflows fp32 (amax below fmax / FLT_MAX) are copied unchanged.
 //
 // The rounding is the hardware minifloat conversion (cvt.rn.satfinite to
 // e2m1x2 / e3m2x2 / e4m3x2 / e5m2x2, then back to f16x2, where every value of
@@ -340,7 +341,9 @@ __global__ void __launch_bounds__(kThreads, kMinCtas) fake_quant_kernel(
         for (int o = 16; o > 0; o >>= 1)
             mbits = max(mbits, __shfl_xor_sync(kFull, mbits, o));
 
-        if (q.f.code == 0 || mbits == 0u || mbits >= 0x7f800000u) {   // kept: bit-for-bit copy
+        // kept (bit-for-bit copy): no format, a zero row, a non-finite value,
+        // or a row so small that its scale factor fmax / amax overflows fp32
+        if (q.f.code == 0 || mbits == 0u || mbits >= 0x7f800000u || isinf(q.f.fmax / __uint_as_float(mbits))) {
             if (q.src != q.dst) {
                 for (int64_t t = lane; t < q.head; t += 32)
                     Act<DT>::copy(q.src, q.dst, t);

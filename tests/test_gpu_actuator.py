@@ -44,9 +44,11 @@ def _oracle_apply(host_in, off, rows, cols, fmt_of_unit):
 
 
 def _special_rows(x, off, rows, cols):
-    """Plant zero, NaN, Inf, -0 and huge-range rows in the first units."""
+    """Plant zero, NaN, Inf, -0, huge-range and tiny rows in the first units
+    (the tiny row's amax, 1e-37, makes fmax / amax overflow fp32 for E4M3
+    and E5M2: that row must come back unchanged, with no NaN)."""
     import torch
-    for b, kind in enumerate(["zero", "nan", "inf", "negzero", "wide"]):
+    for b, kind in enumerate(["zero", "nan", "inf", "negzero", "wide", "tiny"]):
         if b >= len(off) or rows[b] == 0:
             continue
         s, c = int(off[b]), int(cols[b])
@@ -58,9 +60,14 @@ def _special_rows(x, off, rows, cols):
             x[s] = float("-inf")
         elif kind == "negzero":
             x[s:s + c] = -0.0
-        else:
+        elif kind == "wide":
             x[s:s + c] = torch.logspace(-30, 30, c, dtype=torch.float32).to(x.dtype) * \
                 torch.sign(torch.randn(c)).to(x.dtype)
+        else:
+            row = torch.randn(c, dtype=torch.float32) * 1e-37
+            row[::4] = 0.0
+            row[0] = 1e-37
+            x[s:s + c] = row.to(x.dtype)
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])

@@ -101,6 +101,45 @@ def test_per_token_scaling_closed_forms():
     assert np.array_equal(yz[7], oracle.fake_quant(x, oracle.FQ_E2M1)[7])
 
 
+@pytest.mark.parametrize("code", sorted(FORMATS))
+def test_rows_whose_scale_factor_overflows_are_kept(code):
+    """A row with a finite amax below fmax / FLT_MAX would get the scale
+    factor inv = fmax / amax = +inf in fp32, turning its zeros into NaN
+    (0 * inf).  Such a row is kept bit for bit, like a zero row; a row just
+    above that bound is quantized as usual (finite, its max maps back to
+    within one rounding of itself)."""
+    torch = pytest.importorskip("torch")
+    fmax = np.float32(FORMATS[code][4])
+    bound = fmax / np.finfo(np.float32).max             # inv overflows below this amax
+    rng = np.random.default_rng(11)
+    with np.errstate(over="ignore"):
+        _overflow_rows(code, fmax, bound, rng, torch)
+
+
+def _overflow_rows(code, fmax, bound, rng, torch):
+    for amax, kept in ((np.float32(bound * 0.5), True), (np.float32(bound * 4.0), False),
+                       (np.float32(1e-37), bool(np.isinf(np.float32(fmax) / np.float32(1e-37))))):
+        x = (rng.uniform(-1.0, 1.0, (3, 50)) * amax).astype(np.float32)
+        x[:, ::5] = 0.0                                  # zeros that 0 * inf would make NaN
+        x[:, 1] = amax
+        y = oracle.fake_quant(x, code)
+        assert not np.isnan(y).any()
+        if kept:
+            assert np.array_equal(y.view(np.uint32), x.view(np.uint32))
+        else:
+            assert np.all(np.isfinite(y)) and np.all(y[:, ::5] == 0.0)
+            np.testing.assert_allclose(np.max(np.abs(y), axis=1), amax, rtol=1e-6)
+        # the same rows as bf16 bit patterns
+        xb = torch.from_numpy(x).to(torch.bfloat16)
+        bits = xb.view(torch.int16).numpy().view(np.uint16)
+        amax_b = float(xb.abs().max())
+        yb = oracle.fake_quant(bits, code)
+        yf = torch.from_numpy(yb.view(np.int16)).view(torch.bfloat16).float().numpy()
+        assert not np.isnan(yf).any()
+        if np.isinf(np.float32(fmax) / np.float32(amax_b)):
+            assert np.array_equal(yb, bits)
+
+
 def test_bf16_rows():
     torch = pytest.importorskip("torch")
     rng = np.random.default_rng(10)
