@@ -349,18 +349,23 @@ gnmr_status gnmr_actuator_destroy(gnmr_actuator *a);
  * The arena is read as 64 KiB chunks split into contiguous ranges over the
  * GPU's warps, at the step kernel's streaming rate.  A unit outside [0, arena_elems)
  * gives GNMR_ERR_LAYOUT ("unit off arena"); other details: "dtype unknown",
- * "NULL pointer", "arena misalign", "CUDA failed".  The call makes no host
+ * "NULL pointer", "arena misalign", "CUDA failed", "device query" (the
+ * current device or its SM count could not be read).  The call makes no host
  * allocation either, on success or failure.
  *
  * The first call on a device looks up the array's device address for that
  * device; make that first call before any stream capture.  The layout tables
  * are uploaded (pageable host->device copies) only when the layout, dtype or
  * device differs from the previous call's; a call repeating the previous
- * layout enqueues one memset and one kernel, so it may be captured in a CUDA
- * graph.  Every call shares the one array and leaves its contents behind
- * (each call clears what must start at zero); calls that overlap on the GPU
- * race on it, so callers must serialise them (one stream, one thread at a
- * time). */
+ * layout enqueues one memset and one kernel.  Every call shares the one
+ * array and leaves its contents behind (each call clears what must start at
+ * zero); calls that overlap on the GPU race on it, so callers must serialise
+ * them (one stream, one thread at a time).  Each upload tags the tables with
+ * a new generation number and every kernel checks it: a kernel that runs
+ * after another call has replaced the tables with a different layout writes
+ * NaN for every unit instead of norms of the wrong layout.  The array's
+ * address is cached per device for the life of the process: after a
+ * cudaDeviceReset this function must not be called again on that device. */
 gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena_elems, int32_t dtype,
                                    int32_t num_units, const int64_t *offsets,
                                    const int64_t *lengths, double *d_norms, void *stream);

@@ -24,6 +24,7 @@
 #include <mutex>
 
 #include <cuda_runtime.h>
+#include <math_constants.h>
 
 #include "gnmr.h"
 #include "gnmr_internal.h"
@@ -42,7 +43,8 @@ constexpr int kUnroll = 8;                             // 16-byte loads in fligh
 constexpr int kMaxDevices = 64;
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
-constexpr size_t kOffOffsets = 0;
+constexpr size_t kOffGeneration = 0;                   // layout generation of the tables below
+constexpr size_t kOffOffsets = align256(kOffGeneration + 8);
 constexpr size_t kOffLengths = align256(kOffOffsets + 8 * kMaxUnits);
 constexpr size_t kOffStart = align256(kOffLengths + 8 * kMaxUnits);
 constexpr size_t kOffTicket = align256(kOffStart + 8 * (kMaxUnits + 1));
@@ -53,14 +55,15 @@ constexpr size_t kOffPieces = align256(kOffBound + 8 * (kMaxWarps + 1));
 constexpr size_t kOffPartial = align256(kOffPieces + 8 * kMaxUnits);
 constexpr size_t kScratchBytes = align256(kOffPartial + 8 * (kMaxUnits + kMaxWarps));
 
-// All scratch of gnmr_unit_norms_static: unit offsets and lengths (copied from
-// the caller's host arrays), each unit's first chunk index, per-unit tickets,
+// All scratch of gnmr_unit_norms_static: the generation number of the layout
+// the tables hold, unit offsets and lengths (copied from the caller's host arrays), each unit's first chunk index, per-unit tickets,
 // each unit's first partial slot, each warp's first unit and first chunk,
 // each unit's first warp and piece count, and one fp64 partial per
 // (warp, unit) piece.
 static __device__ __align__(256) unsigned char g_norm_scratch[kScratchBytes];
 
 struct View {
+    unsigned long long *generation;
     int64_t *offset;
     int64_t *length;
     int64_t *chunk_start;   // [U + 1]
@@ -74,7 +77,8 @@ struct View {
 
 __host__ __device__ inline View carve(unsigned char *base)
 {
-    return View{reinterpret_cast<int64_t *>(base + kOffOffsets),
+    return View{reinterpret_cast<unsigned long long *>(base + kOffGeneration),
+                reinterpret_cast<int64_t *>(base + kOffOffsets),
                 reinterpret_cast<int64_t *>(base + kOffLengths),
                 reinterpret_cast<int64_t *>(base + kOffStart),
                 reinterpret_cast<uint32_t *>(base + kOffTicket),
@@ -105,15 +109,27 @@ __host__ __device__ inline int64_t unit_chunks(int64_t len, int chunk_shift)
 // segment reduction, adding the chunks of one unit in order; a unit held by
 // one warp is finished there, a unit spread over several by the warp that
 // takes its last ticket, which adds the pieces in slot order.
+//
+// `generation` is the layout generation the call enqueued its work for.  If
+// the tables in the scratch array hold another one (a call with a different
+// layout replaced them before this kernel ran: calls that overlap on the
+// GPU), the kernel writes NaN for every unit instead of reading them.
 template <int DT>
 __global__ void __launch_bounds__(kThreads, 2) static_norms_kernel(const void *arena, unsigned char *base,
                                                                    int32_t num_units, int64_t W,
-                                                                   int64_t chunk_elems, double *norms)
+                                                                   int64_t chunk_elems, double *norms,
+                                                                   unsigned long long generation)
 {
     constexpr int kEB = gnmr::Elem<DT>::kBytes;
     const View v = carve(base);
     const int lane = threadIdx.x & 31;
     const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarpsPerCta + (threadIdx.x >> 5);
+    if (__ldcg(v.generation) != generation) {
+        const int64_t threads = static_cast<int64_t>(gridDim.x) * blockDim.x;
+        for (int64_t u = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < num_units; u += threads)
+            norms[u] = CUDART_NAN;
+        return;
+    }
     if (w >= W)
         return;
     const int64_t c0 = v.bound[w], c1 = v.bound[w + 1];
@@ -184,6 +200,11 @@ __global__ void __launch_bounds__(kThreads, 2) static_norms_kernel(const void *a
             finish(b, wp, s);
             s = 0.0;
             do {
+                if (b + 1 >= num_units) {                // tables not of this layout: stop
+                    if (lane == 0)
+                        norms[b] = CUDART_NAN;
+                    return;
+                }
                 meta(++b);
             } while (c >= next);
         }
@@ -221,6 +242,7 @@ int64_t g_host_pieces[kMaxUnits];
 // units.  Compared element by element, so a match is exact.
 struct Uploaded {
     int device = -1;
+    unsigned long long generation = 0;   // written with the tables to the device scratch
     int sms = 0;
     int32_t dtype = -1;
     int32_t num_units = 0;
@@ -230,6 +252,7 @@ struct Uploaded {
     int64_t lengths[kMaxUnits];
 };
 Uploaded g_uploaded;
+unsigned long long g_next_generation = 1;   // the device scratch starts at 0: no layout
 
 bool same_layout(int dev, int sms, int32_t dtype, int32_t num_units, const int64_t *offsets,
                  const int64_t *lengths)
@@ -271,9 +294,10 @@ constexpr char kErrNull[] = "NULL pointer";
 constexpr char kErrLayout[] = "unit off arena";
 constexpr char kErrArena[] = "arena misalign";
 constexpr char kErrCuda[] = "CUDA failed";
+constexpr char kErrDevice[] = "device query";
 static_assert(sizeof(kErrDtype) <= 16 && sizeof(kErrUnits) <= 16 && sizeof(kErrNull) <= 16 &&
                   sizeof(kErrLayout) <= 16 && sizeof(kErrArena) <= 16 &&
-                  sizeof(kErrCuda) <= 16,
+                  sizeof(kErrCuda) <= 16 && sizeof(kErrDevice) <= 16,
               "failure details must fit a short string");
 
 template <size_t N>
@@ -317,9 +341,10 @@ extern "C" gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena
     unsigned char *base = static_cast<unsigned char *>(addr);
     const View v = carve(base);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    int dev = 0, sms = 1;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+        return reject(GNMR_ERR_CUDA, kErrDevice);
 
     std::lock_guard<std::mutex> lock(g_plan_mu);
     if (!same_layout(dev, sms, dtype, num_units, offsets, lengths)) {
@@ -374,6 +399,10 @@ extern "C" gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena
                 ++u;
             g_host_warp_unit[w] = u;
         }
+        // the generation goes last: a kernel of this call sees it only with
+        // every table of this layout already in place (stream order)
+        static unsigned long long host_generation;
+        host_generation = g_next_generation++;
         e = cudaMemcpyAsync(v.offset, offsets, sizeof(int64_t) * num_units, cudaMemcpyHostToDevice, st);
         if (e == cudaSuccess)
             e = cudaMemcpyAsync(v.length, lengths, sizeof(int64_t) * num_units, cudaMemcpyHostToDevice, st);
@@ -391,8 +420,12 @@ extern "C" gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena
         if (e == cudaSuccess)
             e = cudaMemcpyAsync(v.pieces, g_host_pieces, sizeof(int64_t) * num_units, cudaMemcpyHostToDevice,
                                 st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(v.generation, &host_generation, sizeof host_generation, cudaMemcpyHostToDevice,
+                                st);
         if (e != cudaSuccess)
             return reject(GNMR_ERR_CUDA, kErrCuda);
+        g_uploaded.generation = host_generation;
         std::memcpy(g_uploaded.offsets, offsets, sizeof(int64_t) * num_units);
         std::memcpy(g_uploaded.lengths, lengths, sizeof(int64_t) * num_units);
         g_uploaded.device = dev;
@@ -407,10 +440,11 @@ extern "C" gnmr_status gnmr_unit_norms_static(const void *d_arena, int64_t arena
     if (e != cudaSuccess)
         return reject(GNMR_ERR_CUDA, kErrCuda);
     const int grid = static_cast<int>((W + kWarpsPerCta - 1) / kWarpsPerCta);
+    const unsigned long long gen = g_uploaded.generation;
     if (dtype == GNMR_DTYPE_BF16)
-        static_norms_kernel<1><<<grid, kThreads, 0, st>>>(d_arena, base, num_units, W, chunk_elems, d_norms);
+        static_norms_kernel<1><<<grid, kThreads, 0, st>>>(d_arena, base, num_units, W, chunk_elems, d_norms, gen);
     else
-        static_norms_kernel<0><<<grid, kThreads, 0, st>>>(d_arena, base, num_units, W, chunk_elems, d_norms);
+        static_norms_kernel<0><<<grid, kThreads, 0, st>>>(d_arena, base, num_units, W, chunk_elems, d_norms, gen);
     e = cudaGetLastError();
     if (e != cudaSuccess)
         return reject(GNMR_ERR_CUDA, kErrCuda);

@@ -5,8 +5,9 @@ it, or the deployment fixes its footprint up front).  Its scratch is a static
 device array inside libgnmr, so it needs no handle.
 
 Called through the C ABI and checked against gnmr_step's own norm output
-(stats->norm) on the same arena, twice in a row, within the tolerance of the
-other parity tests.  Kept in its own file, collected last."""
+(stats->norm) and against the oracle on the same bytes, twice in a row,
+within the tolerance of the other parity tests.  Kept in its own file,
+collected last."""
 import numpy as np
 import pytest
 
@@ -32,9 +33,11 @@ def _static_norms(lib, arena, w, out, stream=0):
 def test_static_norms_match_gnmr_step(config, shrink, cuda_device):
     import torch
     lib = N.load()
+    import oracle
     w = workloads.make(config, shrink=shrink, steps=3)
     filler = workloads.Filler(w, cuda_device)
     arena = filler.new_arena()
+    host = torch.empty(arena.numel(), dtype=arena.dtype, pin_memory=True)
     mon = Monitor(w.offsets, w.lengths, device=0, **w.monitor_kwargs())
     stats = mon.new_stats()
     try:
@@ -48,6 +51,11 @@ def test_static_norms_match_gnmr_step(config, shrink, cuda_device):
             torch.cuda.synchronize()
             got = out.cpu().numpy()
             np.testing.assert_allclose(got, want, rtol=RTOL, atol=0)
+            # and against the oracle on the same bytes (Eq. local_gradient, summed in fp64)
+            host.copy_(arena)
+            view = host.view(torch.int16).numpy().view(np.uint16) if w.dtype == "bf16" else host.numpy()
+            exact = oracle.unit_norms_threaded(view, w.offsets, w.lengths, 16)
+            np.testing.assert_allclose(got, exact, rtol=RTOL, atol=0)
     finally:
         mon.close()
 
@@ -112,35 +120,40 @@ def test_static_norms_follow_layout_changes(cuda_device):
     np.testing.assert_allclose(out[:len(off)].cpu().numpy(), oracle.unit_norms(host, off, ln), rtol=RTOL, atol=0)
 
 
-def test_static_norms_repeat_layout_is_graph_capturable(cuda_device):
-    """Once a layout is on the device, a call repeating it enqueues no host
-    copies: it is captured in a CUDA graph, and replays compute the norms of
-    whatever the arena holds at replay time."""
+def test_static_norms_reject_tables_of_another_layout(cuda_device):
+    """Calls that overlap on the GPU race on the shared array.  Here one call
+    repeats the uploaded layout (so it enqueues no upload) behind a long
+    sleep on one stream while a call with a different layout uploads and runs
+    on another stream: when the first kernel finally runs, the tables belong
+    to the other layout, and it writes NaN for every unit instead of reading
+    them.  The second call's norms are correct."""
     import torch
     import oracle
     lib = N.load()
-    rng = np.random.default_rng(22)
+    rng = np.random.default_rng(23)
     n = 1 << 20
-    arena = torch.empty(n, dtype=torch.float32, device=cuda_device)
-    off = np.sort(rng.integers(0, n - 50_000, 64)).astype(np.int64)
-    ln = rng.integers(1, 50_000, 64).astype(np.int64)
-    out = torch.empty(64, dtype=torch.float64, device=cuda_device)
-    stream = torch.cuda.Stream(cuda_device)
-
-    def call():
-        return lib.gnmr_unit_norms_static(arena.data_ptr(), n, N.GNMR_DTYPE_F32, 64, off.ctypes.data,
-                                          ln.ctypes.data, out.data_ptr(), stream.cuda_stream)
-
-    arena.normal_()
-    assert call() == N.GNMR_OK                       # uploads the layout
-    stream.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph, stream=stream):
-        assert call() == N.GNMR_OK
-    for scale in (0.5, 3.0):
-        host = (rng.standard_normal(n) * scale).astype(np.float32)
-        arena.copy_(torch.from_numpy(host))
-        torch.cuda.synchronize()
-        graph.replay()
-        torch.cuda.synchronize()
-        np.testing.assert_allclose(out.cpu().numpy(), oracle.unit_norms(host, off, ln), rtol=RTOL, atol=0)
+    host = rng.standard_normal(n).astype(np.float32)
+    arena = torch.from_numpy(host).to(cuda_device)
+    layouts = []
+    for U in (80, 45):
+        ln = rng.integers(1, 30_000, U).astype(np.int64)
+        off = rng.integers(0, n - 30_000, U).astype(np.int64)
+        layouts.append((off, ln))
+    (off1, ln1), (off2, ln2) = layouts
+    out1 = torch.zeros(80, dtype=torch.float64, device=cuda_device)
+    out2 = torch.zeros(45, dtype=torch.float64, device=cuda_device)
+    s1, s2 = torch.cuda.Stream(cuda_device), torch.cuda.Stream(cuda_device)
+    assert lib.gnmr_unit_norms_static(arena.data_ptr(), n, N.GNMR_DTYPE_F32, 80, off1.ctypes.data,
+                                      ln1.ctypes.data, out1.data_ptr(), s1.cuda_stream) == N.GNMR_OK
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(out1.cpu().numpy(), oracle.unit_norms(host, off1, ln1), rtol=RTOL, atol=0)
+    with torch.cuda.stream(s1):
+        torch.cuda._sleep(200_000_000)               # about 0.1 s on this GPU's clock
+    assert lib.gnmr_unit_norms_static(arena.data_ptr(), n, N.GNMR_DTYPE_F32, 80, off1.ctypes.data,
+                                      ln1.ctypes.data, out1.data_ptr(), s1.cuda_stream) == N.GNMR_OK
+    assert lib.gnmr_unit_norms_static(arena.data_ptr(), n, N.GNMR_DTYPE_F32, 45, off2.ctypes.data,
+                                      ln2.ctypes.data, out2.data_ptr(), s2.cuda_stream) == N.GNMR_OK
+    s2.synchronize()
+    s1.synchronize()
+    np.testing.assert_allclose(out2.cpu().numpy(), oracle.unit_norms(host, off2, ln2), rtol=RTOL, atol=0)
+    assert np.isnan(out1.cpu().numpy()).all()
