@@ -73,17 +73,19 @@ public:
             status_ = cudaErrorNoDevice;
             return;
         }
-        status_ = prev_ == dev ? cudaSuccess : cudaSetDevice(dev);
+        switched_ = prev_ != dev;
+        status_ = switched_ ? cudaSetDevice(dev) : cudaSuccess;
     }
     ~DeviceScope()
     {
-        if (prev_ >= 0)
+        if (switched_)
             cudaSetDevice(prev_);
     }
     cudaError_t status() const { return status_; }
 
 private:
     int prev_ = -1;
+    bool switched_ = false;
     cudaError_t status_ = cudaSuccess;
 };
 
