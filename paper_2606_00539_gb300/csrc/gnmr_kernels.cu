@@ -682,22 +682,59 @@ __device__ void radix_select_cut(const uint64_t *keys, const int32_t *units, uin
     thr_lo = pre_lo;
 }
 
+// Does entry (kj, uj) rank above (k, u)?  Risk descending, then unit ascending.
+__device__ __forceinline__ uint32_t ranks_above(uint64_t kj, int32_t uj, uint64_t k, int32_t u)
+{
+    return (kj > k) | ((kj == k) & (uj < u));
+}
+
 // Commits the r largest (key desc, unit asc) of the n cut-list entries,
-// 1 <= r < n <= kCutCap.  Up to one entry per thread: each entry's rank is
-// counted against all others directly; larger lists use the radix select.
+// 1 <= r < n <= kCutCap.  Each entry's rank is counted against all others
+// directly: up to 32 entries in warp 0's registers (shuffles), up to one per
+// thread from shared memory (eight entries per step, loads issued together);
+// larger lists use the radix select.
 __device__ void select_cut(const StepParams &p, bool stat, uint32_t c, uint32_t n, uint32_t r, const uint64_t *ck,
                            const int32_t *cu, const uint32_t *cl, uint32_t *hist, uint32_t *wsum, uint32_t *misc)
 {
+    if (n <= 32) {
+        if (threadIdx.x < 32) {
+            const uint32_t i = threadIdx.x;
+            const bool mine = i < n;
+            const uint64_t k = mine ? ck[i] : 0ull;
+            const int32_t u = mine ? cu[i] : 0;
+            uint32_t rank = 0;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const uint64_t kj = __shfl_sync(kFull, k, j);
+                const int32_t uj = __shfl_sync(kFull, u, j);
+                rank += (static_cast<uint32_t>(j) < n) ? ranks_above(kj, uj, k, u) : 0u;
+            }
+            if (mine && rank < r)
+                commit_selected(p, stat, u, __longlong_as_double(static_cast<long long>(k)), cl[i]);
+        }
+        return;
+    }
     if (n <= blockDim.x) {
         const uint32_t i = threadIdx.x;
         if (i < n) {
             const uint64_t k = ck[i];
             const int32_t u = cu[i];
             uint32_t rank = 0;
-            for (uint32_t j = 0; j < n; ++j) {
-                const uint64_t kj = ck[j];
-                rank += (kj > k || (kj == k && cu[j] < u)) ? 1u : 0u;
+            uint32_t j = 0;
+            for (; j + 8 <= n; j += 8) {
+                uint64_t kj[8];
+                int32_t uj[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    kj[q] = ck[j + q];
+                    uj[q] = cu[j + q];
+                }
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    rank += ranks_above(kj[q], uj[q], k, u);
             }
+            for (; j < n; ++j)
+                rank += ranks_above(ck[j], cu[j], k, u);
             if (rank < r)
                 commit_selected(p, stat, u, __longlong_as_double(static_cast<long long>(k)), cl[i]);
         }
