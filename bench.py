@@ -492,20 +492,31 @@ def workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budge
         for j in range(K):
             calls[j]()
         stream.synchronize()
-        # pass 1: back-to-back prepared calls, each bracketed by its own events
+        # pass 1: back-to-back prepared calls (one C call per step, nothing
+        # else on the host between them), timed as a region
         mon.set_state(blob, stream)
         wall0 = time.time()
         region[0].record(stream)
+        t_host = time.perf_counter()
+        for j in range(K):
+            calls[j]()
+        t_host = time.perf_counter() - t_host
+        region[1].record(stream)
+        stream.synchronize()
+        per_pass_counts.append(counts.cpu().numpy().copy())
+        rec["arenas"] = f"{K} distinct trace-step arenas, generated before timing"
+        rec["us_per_step"] = us(region[0].elapsed_time(region[1]) / K)
+        rec["host_us_per_call"] = round(t_host / K * 1e6, 1)
+        # pass 1b: the same steps, each bracketed by its own event pair (the
+        # kernel durations; the event records add host time between launches)
+        mon.set_state(blob, stream)
         for j in range(K):
             ev[j][0].record(stream)
             calls[j]()
             ev[j][1].record(stream)
-        region[1].record(stream)
         stream.synchronize()
         per_ms = [a.elapsed_time(b) for a, b in ev]
         per_pass_counts.append(counts.cpu().numpy().copy())
-        rec["arenas"] = f"{K} distinct trace-step arenas, generated before timing"
-        rec["us_per_step"] = us(region[0].elapsed_time(region[1]) / K)
         # pass 2: the K calls captured in one CUDA graph and replayed
         mon.set_state(blob, stream)
         graph = torch.cuda.CUDAGraph()
@@ -592,7 +603,8 @@ def per_workload_records(args, dev, peak, peak_kind) -> dict:
     out = {"peak_gbs": peak, "peak_source": f"{peak_kind} hbm_gbs",
            "what": ("per workload: trace steps t0..t0+K-1 of its own synthetic trace after a fresh monitor "
                     "ran steps 1..t0-1; us_per_step = back-to-back prepared calls (distinct arenas) or the "
-                    "kernel mean (regenerated arenas); kernel_us_* from per-step CUDA events; gbs and frac "
+                    "kernel mean (regenerated arenas); host_us_per_call = host time of one prepared call; "
+                    "kernel_us_* from per-step CUDA events; gbs and frac "
                     "from the kernel mean; candidates = |C_t| over the timed steps")}
     try:
         for n in names:
