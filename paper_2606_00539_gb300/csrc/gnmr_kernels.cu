@@ -13,20 +13,25 @@
 // Phase 2, the warp that completes unit b.  A unit split over several warps
 // collects their partial sums through fixed slots and a per-unit ticket; the
 // warp that takes the last ticket sums the slots in slot order (so the result
-// does not depend on timing).  Completed units queue up in the warp's lanes
-// and run the unit epilogue 32 at a time, one unit per lane: Algorithm 1
-// (GNMR, Delta-GNMR, incremental mean, window queue), the combined risk
+// does not depend on timing); a unit of two parts trades its partial in one
+// atomic exchange.  Completed units queue up in the warp's lanes and run the
+// unit epilogue 32 at a time, one unit per lane: Algorithm 1 (GNMR,
+// Delta-GNMR, incremental mean, window queue), the combined risk
 // R = max{GNMR/alpha_t, Delta-GNMR/beta_t} and the candidate test
-// R > 1 or Lock > 0 (Sec. 3.3), appending candidates to a compact list and
-// writing every unit's outcome if it is not selected.
+// R > 1 or Lock > 0 (Sec. 3.3).  Candidates go to a compact list; members of
+// the capped pool also count in a global risk histogram and, at or above the
+// bin predicted from the previous step's cut, go to a short hot list.  Every
+// unit's outcome if it is not selected is written here.
 //
-// Phase 3, the last CTA to finish (grid ticket).  Top_maxO over the
-// candidate list by an in-CTA radix select on the 96-bit key
-// (R descending, unit index ascending), run on a shared-memory copy of the
-// candidates' keys, then the lock bookkeeping of Algorithm 2 for the
-// selected units, the counts, and the reset of the counters for the next
-// launch.  No CTA ever waits for another: the tickets decide who continues,
-// so the kernel cannot hang whatever the grid size or residency.
+// Phase 3, the last CTA to finish (grid ticket): Top_maxO.  The histogram
+// gives the bin that holds the maxO-th largest risk; one read of the hot list
+// (or, if the prediction missed, of the whole list) commits every candidate
+// above that bin, and the bin's own members are ranked on the 96-bit key
+// (R descending, unit index ascending) in shared memory.  Then the lock
+// bookkeeping of Algorithm 2 for the selected units, the counts, and the
+// reset of the counters for the next launch.  No CTA ever waits for another:
+// the tickets decide who continues, so the kernel cannot hang whatever the
+// grid size or residency.
 //
 // The same kernel also runs either half of a sharded step: phase 1 alone
 // (per-unit sums of squares of a shard) or phases 2-3 alone on sums that the
@@ -778,6 +783,19 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
     } else if (stat && t > p.static_warmup + 1) {
         m = 0;
         n_sel = static_cast<uint32_t>(p.static_keep);
+    } else if (!admission && m <= (stat ? static_cast<uint32_t>(p.static_keep) : static_cast<uint32_t>(p.max_o))) {
+        // every candidate is in the pool and the pool fits the budget: one read of the
+        // list commits all of it and empties the histogram bins it filled (no scan)
+        for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+            double r;
+            int32_t b;
+            uint32_t lk;
+            load_candidate(p.cand + i, r, b, lk);
+            commit_selected(p, stat, b, r, lk);
+            __stcg(p.risk_hist + risk_bin(risk_key(r)), 0u);
+        }
+        n_sel = m;
+        next_hot = 0;                                // a small pool: every candidate is hot next step
     } else {
         const uint32_t cap = stat ? static_cast<uint32_t>(p.static_keep) : static_cast<uint32_t>(p.max_o);
         scan_risk_hist(p, cap, 3 * cap + 64, misc, hist);
