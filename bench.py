@@ -383,14 +383,17 @@ def trigger_sparsity(w, filler, arena, dev) -> dict:
     """Table 3's statistic on the workload's synthetic trace: a fresh monitor
     runs steps 1..T of the trace (untimed, after the timed region) and the
     share of (recoverable unit, step) pairs over each threshold is counted,
-    with the candidate and selected counts of Algorithm 2."""
+    with the candidate and selected counts of Algorithm 2.  Table 11's two
+    trigger statistics come with it: the promotion ratio (selected
+    (unit, step) pairs over all of them) and the hit-maxO rate, read as the
+    share of steps at which |A_t| reached the budget maxO."""
     import torch
     from paper_2606_00539_gb300 import Monitor
     mon = Monitor(w.offsets, w.lengths, device=dev.index, **w.monitor_kwargs())
     stats = mon.new_stats()
     mask = torch.empty(w.num_units, dtype=torch.uint8, device=dev)
     rec = np.asarray(w.recoverable, np.uint8)
-    over_g = over_d = cand = sel = 0
+    over_g = over_d = cand = sel = hit = 0
     try:
         for t in range(w.steps):
             filler.fill(arena, t)
@@ -400,6 +403,7 @@ def trigger_sparsity(w, filler, arena, dev) -> dict:
             g, d = exceedance_counts(stats["gnmr"].cpu().numpy(), stats["dgnmr"].cpu().numpy(), rec, a_t, b_t)
             c = stats["counts"].cpu().tolist()
             over_g, over_d, cand, sel = over_g + g, over_d + d, cand + c[0], sel + c[1]
+            hit += int(w.max_o > 0 and c[1] >= w.max_o)
     finally:
         mon.close()
     pairs = max(1, int(rec.sum()) * w.steps)
@@ -408,6 +412,8 @@ def trigger_sparsity(w, filler, arena, dev) -> dict:
             "candidates_per_step": round(cand / w.steps, 2),
             "selected_per_step": round(sel / w.steps, 2),
             "selected_pct": round(100.0 * sel / pairs, 4),
+            "promotion_ratio": round(sel / pairs, 6),
+            "hit_max_o_rate": round(hit / w.steps, 4),
             "steps": w.steps, "recoverable_units": int(rec.sum()),
             "trace": "the workload's synthetic trace, steps 1..T, one fresh monitor, untimed"}
 

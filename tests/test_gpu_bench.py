@@ -33,6 +33,8 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(clocks)
     sparsity = line["trigger_sparsity"]
     assert sparsity["steps"] > 0 and 0 <= sparsity["selected_pct"] <= 100
+    assert sparsity["promotion_ratio"] == pytest.approx(sparsity["selected_pct"] / 100, abs=1e-5)
+    assert 0 <= sparsity["hit_max_o_rate"] <= 1
     assert cpu["single_thread"]["cores"] == 1 and cpu["single_thread"]["value"] > 0
     per = line["per_workload"]
     assert set(per) >= {"tiny", "aq-stress", "peak_gbs"}

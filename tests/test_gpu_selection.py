@@ -72,11 +72,11 @@ CASES = {
 }
 
 
-def _drive(risks_per_step, policy=0, **policy_kw):
+def _drive(risks_per_step, policy=0, max_o=MAX_O, **policy_kw):
     """Step 1 with n = 1, then one step per entry of risks_per_step (the
     target R of every unit: n = R * A_b with A_b read from the oracle)."""
     import torch
-    kw = dict(window=8, max_o=MAX_O, lock_len=LOCK, eps=0.0)
+    kw = dict(window=8, max_o=max_o, lock_len=LOCK, eps=0.0)
     mon = Monitor(np.zeros(U, np.int64), np.zeros(U, np.int64), dtype="f32", device=0,
                   alpha=1.0, beta=1e6, policy=policy, **kw, **policy_kw)
     ctl = oracle.Controller(U, alpha=(1.0, 1.0), beta=(1e6, 1e6), policy=policy, **kw, **policy_kw)
@@ -156,6 +156,16 @@ def test_admission_cap_counts_only_new_units(cuda_device):
     rng = np.random.default_rng(8)
     steps = [_spread(rng) for _ in range(4)]
     _drive(steps, policy=oracle.POLICY_ADMISSION_CAP)
+
+
+def test_admission_cap_retained_past_the_hot_list_capacity(cuda_device):
+    """Admission cap with a budget of 5,000: the admitted units stay active
+    (their locks keep them candidates), so by the fourth step more than
+    8,192 retained units have to join the hot list, which overflows; the
+    selection then reads the whole candidate list."""
+    rng = np.random.default_rng(10)
+    res = _drive([_spread(rng) for _ in range(5)], policy=oracle.POLICY_ADMISSION_CAP, max_o=5000)
+    assert res.n_selected > 8192
 
 
 def test_static_policy_ranks_by_gnmr_sum(cuda_device):
