@@ -891,6 +891,12 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
     constexpr int kEB = Elem<DT>::kBytes;
     const int lane = threadIdx.x & 31;
     const int warp = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
+    // Launched as a programmatic dependent of whatever precedes it on the
+    // stream: wait here until that kernel has completed and its writes are
+    // visible (the arena, the previous step's state), then let the next step
+    // launch as soon as it finds room on an SM (it waits here too).
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (MODE == kStepFinish) {
         const int64_t t = __ldcg(&p.ctl->steps) + 1;
@@ -1001,11 +1007,19 @@ template <int MODE, int V>
 cudaError_t launch_mode(const StepParams &p, int dtype, int num_ctas, cudaStream_t stream)
 {
     constexpr size_t smem = MODE == kStepPartials ? 0 : kKeyCacheBytes;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(num_ctas));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     if (dtype == 1)
-        gnmr_step_kernel<1, MODE, V><<<num_ctas, kThreads, smem, stream>>>(p);
-    else
-        gnmr_step_kernel<0, MODE, V><<<num_ctas, kThreads, smem, stream>>>(p);
-    return cudaGetLastError();
+        return cudaLaunchKernelEx(&cfg, gnmr_step_kernel<1, MODE, V>, p);
+    return cudaLaunchKernelEx(&cfg, gnmr_step_kernel<0, MODE, V>, p);
 }
 
 template <int V>
