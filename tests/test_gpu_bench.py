@@ -49,4 +49,6 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
         assert rec["frac"] == pytest.approx(rec["gbs"] / per["peak_gbs"], abs=1e-3)
         assert 0 <= rec["selected_mean"] <= rec["max_o"] and rec["candidates_max"] >= 0
         assert {"sm_mhz", "reasons"} <= set(rec["clocks"])
+        assert rec["trace_candidates_mean"] >= 0 and 0 <= rec["trace_selected_mean"] <= rec["max_o"]
+        assert 0 <= rec["trace_hit_max_o_rate"] <= 1
     assert per["aq-stress"]["candidates_mean"] > per["aq-stress"]["max_o"]   # the contended top-k
