@@ -584,3 +584,36 @@ def test_cuda_graph_replay_advances_steps(cuda_device):
             TD.compare(norms, res, got, RTOL)
     finally:
         tr.close()
+
+
+@pytest.mark.parametrize("config,shrink", [("aq-stress", 8), ("llama2-13b", 16)])
+def test_steps_wait_for_the_kernel_that_writes_the_arena(config, shrink, cuda_device):
+    """Steps enqueued right behind the kernel that writes their arena, with no
+    host synchronisation in between: fill, step, fill, step, ... on one
+    stream.  Each step must see its own step's gradients (its norms equal the
+    oracle's on that step's bytes, regenerated separately afterwards), so a
+    step never starts reading before the writer has finished."""
+    import torch
+    import oracle
+    w = workloads.make(config, shrink=shrink, steps=6)
+    filler = workloads.Filler(w, cuda_device)
+    arena = filler.new_arena()
+    mon = _monitor(w)
+    norms = torch.empty((w.steps, w.num_units), dtype=torch.float64, device=cuda_device)
+    stats = mon.new_stats()
+    try:
+        torch.cuda.synchronize()
+        for t in range(w.steps):
+            filler.fill(arena, t)                    # torch's current stream, then the step on it
+            mon.step(arena, stats=dict(stats, norm=norms[t]))
+        torch.cuda.synchronize()
+        got = norms.cpu().numpy()
+        check = filler.new_arena()
+        for t in range(w.steps):
+            filler.fill(check, t)
+            host = check.cpu()
+            view = host.view(torch.int16).numpy().view(np.uint16) if w.dtype == "bf16" else host.numpy()
+            want = oracle.unit_norms_threaded(view, w.offsets, w.lengths, 8)
+            np.testing.assert_allclose(got[t], want, rtol=RTOL, atol=0, err_msg=f"step {t + 1}")
+    finally:
+        mon.close()
