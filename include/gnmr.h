@@ -201,7 +201,11 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out);
  *   stream       cudaStream_t as void*; NULL = legacy default stream.
  *   d_mask       device uint8 [num_units], written (1 = recovery path).
  *   stats        optional statistics outputs (see gnmr_stats), or NULL.
- * The arena must not change until the stream has passed the step.  Errors:
+ * The arena must not change until the stream has passed the step.  The
+ * kernel is launched as a programmatic dependent of the work before it on
+ * the stream: it may be scheduled early, but it waits before its first
+ * memory access until that work has completed and its writes are visible,
+ * so stream order holds as for a plain launch.  Errors:
  * GNMR_ERR_INVALID_ARG, GNMR_ERR_LAYOUT, GNMR_ERR_STATE, GNMR_ERR_CUDA (the
  * launch failed). */
 gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems,
