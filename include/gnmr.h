@@ -222,15 +222,16 @@ gnmr_status gnmr_step(gnmr_handle *h, const void *d_arena, int64_t arena_elems,
  * [num_units]); it changes no controller state.  The caller then sums d_sumsq
  * across ranks (e.g. an all-reduce) and calls gnmr_finish on every rank:
  * identical sums give identical masks everywhere.  Arguments and errors as
- * gnmr_step (d_sumsq replaces d_mask). */
+ * gnmr_step (d_sumsq replaces d_mask).  Launched as gnmr_step is (a
+ * programmatic dependent that waits for the preceding work first). */
 gnmr_status gnmr_step_partials(gnmr_handle *h, const void *d_arena, int64_t arena_elems,
                                void *stream, double *d_sumsq);
 
 /* Sharded step, second half: one controller step (Algorithms 1 and 2, as in
  * gnmr_step from step 2 on) on given per-unit sums of squares: n_b =
  * sqrt(d_sumsq[b]).  d_sumsq: device fp64 [num_units], read only.  d_mask and
- * stats as in gnmr_step.  Advances the step counter.  Errors:
- * GNMR_ERR_INVALID_ARG, GNMR_ERR_STATE, GNMR_ERR_CUDA. */
+ * stats as in gnmr_step.  Advances the step counter.  Launched as gnmr_step
+ * is.  Errors: GNMR_ERR_INVALID_ARG, GNMR_ERR_STATE, GNMR_ERR_CUDA. */
 gnmr_status gnmr_finish(gnmr_handle *h, const double *d_sumsq, void *stream, uint8_t *d_mask,
                         const gnmr_stats *stats);
 
