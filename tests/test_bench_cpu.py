@@ -117,3 +117,20 @@ def test_host_arena_follows_the_layout_and_the_trace_scales():
     bits = h[b.offsets[1]:b.offsets[1] + b.lengths[1]].astype(np.uint32) << 16
     vals = bits.view(np.float32)
     assert np.all(np.isfinite(vals)) and np.all(vals != 0)
+
+
+def test_both_arms_print_the_same_config():
+    """The reference arm's config object is the one the GPU arm prints for
+    the same workload and arguments (the driver compares the two)."""
+    import io
+    import contextlib
+    import workloads
+    out = io.StringIO()
+    with contextlib.redirect_stdout(out):
+        bench.main(["--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "0"])
+    line = json.loads(out.getvalue().strip().splitlines()[-1])
+    args = bench.parse_args(["--workload", "tiny", "--steps", "1", "--warmup", "0"])
+    want = bench.workload_config(workloads.make("tiny"), args, args.arenas, 1)
+    assert line["config"] == want
+    assert "every step the whole 64-unit tiny layout" in line["cpu_baseline"]["sample"]
+    assert "note" not in line                          # the full layout, not a sample
