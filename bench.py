@@ -447,8 +447,9 @@ def workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budge
     trace's own candidate pools and selections.  Arenas that fit in
     `budget_bytes` are all generated first (passes: back-to-back prepared
     calls with per-step events, one CUDA graph of the K calls, and, for
-    arenas under 2 GB, an L2 flush before every step; the graph pass reports
-    the better of two timed replays); larger ones are
+    arenas under 2 GB, an L2 flush (a 512 MB write) before every step, and an
+    L2 clean (a 512 MB read, no dirty lines left) before every step; the graph
+    pass reports the better of two timed replays); larger ones are
     regenerated between steps, outside each step's events, followed by a
     512 MB read so the step starts with no dirty or arena lines in L2."""
     import torch
@@ -563,7 +564,19 @@ def workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budge
             fl = [a.elapsed_time(b) for a, b in ev]
             per_pass_counts.append(counts.cpu().numpy().copy())
             rec["l2_flushed_us_mean"] = us(statistics.mean(fl))
-            del flush
+            # the same with L2 emptied by a 512 MB read: no dirty lines left to
+            # write back during the step, so this is the cost of cold state alone
+            clean_out = torch.empty((), dtype=torch.int64, device=dev)
+            mon.set_state(blob, stream)
+            for j in range(K):
+                torch.sum(flush, dim=0, dtype=torch.int64, out=clean_out)
+                ev[j][0].record(stream)
+                calls[j]()
+                ev[j][1].record(stream)
+            stream.synchronize()
+            per_pass_counts.append(counts.cpu().numpy().copy())
+            rec["l2_cleaned_us_mean"] = us(statistics.mean(a.elapsed_time(b) for a, b in ev))
+            del flush, clean_out
         wall1 = time.time()
         del calls, arenas
     else:

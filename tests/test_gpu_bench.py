@@ -43,7 +43,7 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
         assert rec["steps"] == steps and rec["trace_steps"][1] - rec["trace_steps"][0] + 1 == steps
         assert rec["warmup_steps"] >= 3 and rec["passes_agree"] is True
         for key in ("us_per_step", "kernel_us_mean", "kernel_us_min", "graph_us_per_step",
-                    "l2_flushed_us_mean"):
+                    "l2_flushed_us_mean", "l2_cleaned_us_mean"):
             assert rec[key] > 0, key
         assert rec["kernel_us_min"] <= rec["kernel_us_mean"] <= rec["kernel_us_max"]
         assert rec["frac"] == pytest.approx(rec["gbs"] / per["peak_gbs"], abs=1e-3)
