@@ -5,8 +5,8 @@
 // segments of the arena).  For every segment piece in its run it streams the
 // gradient with 16-byte read-only loads (8 or 16 in flight per lane, by the
 // loop shape), squares in fp32, sums blocks of 16 iterations in fp32 and the
-// blocks as float pairs (error-free TwoSum), and all-reduces the pairs across
-// the warp with shuffles, converting to fp64 once per segment:
+// blocks as float pairs (error-free TwoSum), and all-reduces the lanes' totals
+// across the warp with shuffles, converting to fp64 once per segment:
 // n_b = ||g_b||_2 (Sec. 2, Eq. local_gradient).  No shared memory, no block
 // barrier on this path.  (The streaming reduction lives in gnmr_stream.cuh.)
 //

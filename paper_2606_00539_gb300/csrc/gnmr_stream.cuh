@@ -5,8 +5,9 @@
 // A warp reads a segment with 16-byte loads on the non-coherent path (no L1
 // allocation, 256-byte L2 prefetch), squares in fp32, sums short blocks in
 // fp32 and the blocks as an unevaluated pair of floats (hi + lo, about 48
-// significant bits), reduces the pairs across the warp the same way, and
-// converts to fp64 once per segment.  It flags segments whose fp32 squares
+// significant bits), then adds the 32 lanes' totals with an fp32 xor
+// butterfly (non-negative terms: at most five roundings, about 3e-7
+// relative) and converts to fp64 once per segment.  It flags segments whose fp32 squares
 // may have lost accuracy (denormal or overflowing squares), which the caller
 // recomputes with exact fp64 squares.  Any element alignment: a scalar head
 // and tail around the 16-byte body.
@@ -15,7 +16,10 @@
 // the SM retires one fp64 warp-instruction every 20 cycles, shared by all its
 // warps.  A five-round fp64 shuffle reduction per segment held that pipe 40 %
 // of the time on layouts of many small units and stalled the streams; the
-// fp32 error-free additions run on the fp32 pipe.
+// fp32 error-free additions run on the fp32 pipe.  The pairs keep a long run
+// of blocks accurate; the final five-level tree over the lanes does not need
+// them (measured: a pair-wise TwoSum butterfly there cost 1 us more on 100K
+// units).
 #ifndef GNMR_STREAM_CUH
 #define GNMR_STREAM_CUH
 
@@ -137,24 +141,6 @@ __device__ __forceinline__ void pair_add(float &hi, float &lo, float x)
     lo = __fadd_rn(lo, e);
 }
 
-// Sum of the lanes' pairs (xor butterfly): both partners combine the same
-// two pairs with commutative operations, so every lane ends with the same
-// bits.  Returns hi + lo in fp64; hi_out = the pair's leading float.
-__device__ __forceinline__ double warp_allreduce_pair(float hi, float lo, float &hi_out)
-{
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float ohi = __shfl_xor_sync(kFull, hi, o);
-        const float olo = __shfl_xor_sync(kFull, lo, o);
-        float s, e;
-        two_sum(hi, ohi, s, e);
-        hi = s;
-        lo = __fadd_rn(__fadd_rn(lo, olo), e);
-    }
-    hi_out = hi;
-    return static_cast<double>(hi) + static_cast<double>(lo);
-}
-
 // Sum of squares of n elements at seg, by the whole warp.  Returns the sum
 // in every lane and sets `suspect` when fp32 squaring may have lost accuracy:
 // a nonzero segment whose sum is below 2^-100 (denormal squares) or above
@@ -229,8 +215,14 @@ __device__ __forceinline__ double warp_segment_sumsq(const char *seg, int64_t n,
         blk += a;
     }
     pair_add(acc_hi, acc_lo, blk);
-    float lead;
-    const double acc = warp_allreduce_pair(acc_hi, acc_lo, lead);
+    // the lanes' totals (non-negative) summed by an fp32 xor butterfly: both
+    // partners add the same two operands, so every lane ends with the same bits
+    float tot = acc_hi + acc_lo;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        tot += __shfl_xor_sync(kFull, tot, o);
+    const float lead = tot;
+    const double acc = static_cast<double>(tot);
     bits = __reduce_or_sync(kFull, bits);
     suspect = (bits & Elem<DT>::kMagnitude) != 0u && !(lead >= 0x1p-100f && lead <= 0x1p+100f);
     return acc;
