@@ -207,6 +207,15 @@ def profiled_traffic(paths, workload: str = "llama2-13b"):
     return int(rec["traffic_bytes_per_launch"])
 
 
+def grid_text(info) -> str:
+    """Launch geometry of a handle, from gnmr_get_info."""
+    if info["loop_shape"] == 2:
+        return (f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, {info['num_runs']} runs "
+                f"taken dynamically by {info['num_warps']} warps, large-unit loop shape")
+    return (f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, {info['num_warps']} warp runs, "
+            f"small-unit loop shape")
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -468,8 +477,7 @@ def workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budge
     distinct = K * arena_bytes <= budget_bytes
     rec = {"trace_steps": [t0, t0 + K - 1], "steps": K, "warmup_steps": t0 - 1,
            "units": w.num_units, "dtype": w.dtype, "bytes_per_step": w.grad_bytes,
-           "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, {info['num_warps']} warp runs, "
-                   f"{'large-unit' if info['loop_shape'] == 2 else 'small-unit'} loop shape"}
+           "grid": grid_text(info)}
     def fill(arena, i):
         filler.fill(arena, i)                       # on the current stream: `stream`
 
@@ -615,7 +623,8 @@ def workload_record_on(stream, name, k_steps, w_steps, dev, peak, sampler, budge
         "trace_candidates_mean": round(float(whole[:, 0].mean()), 1),
         "trace_selected_mean": round(float(whole[:, 1].mean()), 2),
         "trace_hit_max_o_rate": round(float(np.mean(whole[:, 1] >= w.max_o)), 4) if w.max_o > 0 else 0.0,
-        "kernel_us_mean": us(kern), "kernel_us_min": us(min(per_ms)), "kernel_us_max": us(max(per_ms)),
+        "kernel_us_mean": us(kern), "kernel_us_median": us(statistics.median(per_ms)),
+        "kernel_us_min": us(min(per_ms)), "kernel_us_max": us(max(per_ms)),
         "gbs": round(w.grad_bytes / (kern / 1e3) / 1e9, 1),
         "frac": round(w.grad_bytes / (kern / 1e3) / 1e9 / peak, 4),
         "candidates_mean": round(float(c[:, 0].mean()), 1), "candidates_max": int(c[:, 0].max()),
@@ -859,9 +868,7 @@ def run_gnmr(args):
             "config": workload_config(w, args, n_arenas, world),
             "launch": {"how": ("one CUDA graph of the timed steps, replayed" if args.graph
                                else "one prepared gnmr_step call per step"),
-                       "grid": f"{info['num_ctas']} CTAs x {info['threads_per_cta']} threads, "
-                               f"{info['num_warps']} warp runs, "
-                               f"{'large-unit' if info['loop_shape'] == 2 else 'small-unit'} loop shape"},
+                       "grid": grid_text(info)},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4),
                          "traffic": traffic if args.shrink == 1 and args.group == "tensor" else None,
@@ -869,6 +876,7 @@ def run_gnmr(args):
                          "algorithmic_bytes": w.grad_bytes,
                          "peak_source": f"{peak_kind} hbm_gbs", "kernel": f"gnmr_step_kernel<{w.dtype}>",
                          "kernel_ms_mean": round(kern_ms, 4),
+                         "kernel_ms_median": round(statistics.median(per_ms), 4),
                          "kernel_ms_min": round(min(per_ms), 4)},
             "cpu_baseline": cpu,
             "e2e": e2e,

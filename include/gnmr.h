@@ -88,8 +88,10 @@ typedef struct gnmr_config {
      * generic-memory-bound), host [num_units], copied; NULL = no Delta M_t. */
     const double *unit_cost;
     /* Shape of the kernel's streaming loop (gnmr_loop_shape).  The shapes
-     * split the arena into different warp runs, so norms agree within
-     * rounding, not bitwise; each shape is bitwise reproducible run to run.
+     * split the arena into different runs, so norms agree within rounding,
+     * not bitwise; each shape is bitwise reproducible call to call (the
+     * large-unit shape hands its runs to warps dynamically, but a run's
+     * partial sum has a fixed slot and a unit's slots are added in order).
      * Default GNMR_LOOP_AUTO. */
     int32_t loop_shape;
 } gnmr_config;
@@ -148,13 +150,16 @@ typedef struct gnmr_info {
     int32_t device;
     int32_t num_ctas;          /* CTAs per gnmr_step launch */
     int32_t threads_per_cta;
-    int32_t num_warps;         /* warps with a non-empty work run */
-    int64_t num_partials;      /* per-(warp, unit) partial sums */
+    int32_t num_warps;         /* warps with a work run */
+    int64_t num_partials;      /* per-(run, unit) partial sums */
     int64_t device_bytes;      /* library-owned device memory */
     int64_t arena_elems_min;   /* max over units of offset + length */
     int64_t steps;             /* gnmr_step calls enqueued so far */
     int32_t loop_shape;        /* gnmr_loop_shape in use (never GNMR_LOOP_AUTO) */
-    int32_t reserved;
+    int32_t num_runs;          /* work runs: one per warp with the small-unit loop;
+                                  about 16 per warp with the large-unit loop, where
+                                  each warp starts on its own and then takes the
+                                  next untaken one */
 } gnmr_info;
 
 typedef struct gnmr_handle gnmr_handle;
@@ -275,10 +280,12 @@ const char *gnmr_status_string(gnmr_status s);
  * create on this thread); never NULL. */
 const char *gnmr_last_error(const gnmr_handle *h);
 
-/* Host-only query of the work partition that gnmr_create would plan: the
- * concatenation of all units (an empty unit counts as one element of work)
- * is cut into at most max_warps contiguous runs of about equal cost
- * (element bytes plus a fixed per-unit cost), one run per warp.  Outputs,
+/* Host-only query of the work partition that gnmr_create plans for the
+ * small-unit loop shape (max_warps = the resident warps): the concatenation
+ * of all units (an empty unit counts as one element of work) is cut into at
+ * most max_warps contiguous runs of about equal cost (element bytes plus a
+ * fixed per-unit cost), one run per warp.  (The large-unit shape cuts the
+ * same way into about 16 runs per warp, see gnmr_info.num_runs.)  Outputs,
  * caller-allocated: run_unit / run_pos [max_warps + 1] (run w covers
  * (run_unit[w], run_pos[w]) up to, not including, (run_unit[w+1],
  * run_pos[w+1])), first_warp / num_parts [num_units] (the warps touching

@@ -82,7 +82,7 @@ class gnmr_info(ctypes.Structure):
         ("arena_elems_min", ctypes.c_int64),
         ("steps", ctypes.c_int64),
         ("loop_shape", ctypes.c_int32),
-        ("reserved", ctypes.c_int32),
+        ("num_runs", ctypes.c_int32),
     ]
 
 

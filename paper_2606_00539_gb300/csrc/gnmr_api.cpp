@@ -23,7 +23,8 @@ struct gnmr_handle {
     int32_t num_ctas = 0;
     int32_t finish_ctas = 0;      // grid of the controller-only launch
     int32_t variant = 0;          // streaming-loop shape (gnmr::kVariant*)
-    int32_t num_warps = 0;
+    int32_t num_warps = 0;        // warps with a first run
+    int32_t num_runs = 0;
     int64_t num_segments = 0;
     int64_t num_partials = 0;
     int64_t device_bytes = 0;
@@ -162,11 +163,11 @@ gnmr_status gnmr_plan_partition(int32_t num_units, const int64_t *lengths, int32
     } catch (const std::bad_alloc &) {
         return GNMR_ERR_OOM;
     }
-    *num_warps = plan.num_warps;
-    for (int32_t w = 0; w <= plan.num_warps; ++w)
+    *num_warps = plan.num_runs;
+    for (int32_t w = 0; w <= plan.num_runs; ++w)
         run_unit[w] = static_cast<int32_t>(plan.run_seg[w]);
-    std::memcpy(run_pos, plan.run_pos.data(), sizeof(int64_t) * (plan.num_warps + 1));
-    std::memcpy(first_warp, plan.first_warp.data(), sizeof(int32_t) * num_units);
+    std::memcpy(run_pos, plan.run_pos.data(), sizeof(int64_t) * (plan.num_runs + 1));
+    std::memcpy(first_warp, plan.first_run.data(), sizeof(int32_t) * num_units);
     std::memcpy(num_parts, plan.num_parts.data(), sizeof(int32_t) * num_units);
     return GNMR_OK;
 }
@@ -286,13 +287,28 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
                 seg_unit[u] = u;
         }
         const int64_t S = static_cast<int64_t>(seg_off.size());
+        // The small-unit loop plans one run per resident warp.  The large-unit
+        // loop plans about kRunsPerWarp runs per warp (never fewer runs than
+        // the one-per-warp plan), which the warps take dynamically.
+        const int64_t grid_warps = int64_t(sms) * per_sm * gnmr::kWarpsPerCta;
+        int64_t max_runs = grid_warps;
+        if (variant == gnmr::kVariantBulk) {
+            const int64_t cost = grad_bytes + U * gnmr::kUnitCostBytes;
+            int64_t run = cost / (grid_warps * gnmr::kRunsPerWarp);
+            run = std::min(std::max(run, gnmr::kBulkRunMin), gnmr::kBulkRunMax);
+            max_runs = std::max(max_runs, (cost + run - 1) / run);
+            if (max_runs > INT32_MAX / 2) {
+                delete h;
+                return fail_create(GNMR_ERR_INVALID_ARG, "work partition failed (too many runs)");
+            }
+        }
         gnmr::Plan plan;
         if (!gnmr::plan_partition(S, seg_len.data(), seg_unit.data(), c.num_units, eb,
-                                  sms * per_sm * gnmr::kWarpsPerCta, plan)) {
+                                  static_cast<int32_t>(max_runs), plan)) {
             delete h;
             return fail_create(GNMR_ERR_INVALID_ARG, "work partition failed (sizes out of range)");
         }
-        const int64_t W = plan.num_warps;
+        const int64_t W = plan.num_runs;
         Carver cv;
         const size_t o_off = cv.take(sizeof(int64_t) * S);
         const size_t o_len = cv.take(sizeof(int64_t) * S);
@@ -328,7 +344,7 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
             std::memcpy(&img[o_cost], c.unit_cost, sizeof(double) * U);
         std::memcpy(&img[o_run_seg], plan.run_seg.data(), sizeof(int64_t) * (W + 1));
         std::memcpy(&img[o_run_pos], plan.run_pos.data(), sizeof(int64_t) * (W + 1));
-        std::memcpy(&img[o_first], plan.first_warp.data(), sizeof(int32_t) * U);
+        std::memcpy(&img[o_first], plan.first_run.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_parts], plan.num_parts.data(), sizeof(int32_t) * U);
         std::memcpy(&img[o_pbase], plan.part_base.data(), sizeof(int64_t) * U);
         std::memset(&img[o_partial], 0xff, sizeof(double) * plan.num_partials);   // every slot empty
@@ -361,7 +377,7 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         p.recoverable = reinterpret_cast<const uint8_t *>(base + o_rec);
         p.run_seg = reinterpret_cast<const int64_t *>(base + o_run_seg);
         p.run_pos = reinterpret_cast<const int64_t *>(base + o_run_pos);
-        p.first_warp = reinterpret_cast<const int32_t *>(base + o_first);
+        p.first_run = reinterpret_cast<const int32_t *>(base + o_first);
         p.num_parts = reinterpret_cast<const int32_t *>(base + o_parts);
         p.part_base = reinterpret_cast<const int64_t *>(base + o_pbase);
         p.partial = reinterpret_cast<double *>(base + o_partial);
@@ -380,7 +396,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         p.static_warmup = c.static_warmup_steps;
         p.static_keep = static_cast<int32_t>(std::min<double>(std::ceil(c.static_fraction * num_rec), num_rec));
         p.num_units = c.num_units;
-        p.num_warps = plan.num_warps;
+        const int32_t warps = static_cast<int32_t>(std::min<int64_t>(plan.num_runs, grid_warps));
+        p.num_warps = warps;
+        p.num_runs = plan.num_runs;
         p.window = c.window;
         p.max_o = c.max_o;
         p.lock_len = c.lock_len;
@@ -401,8 +419,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         h->variant = variant;
         h->num_units = c.num_units;
         h->elem_bytes = eb;
-        h->num_warps = plan.num_warps;
-        h->num_ctas = (plan.num_warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
+        h->num_warps = warps;
+        h->num_runs = plan.num_runs;
+        h->num_ctas = (warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
         {
             const int64_t warps = (U + 31) / 32;
             const int64_t ctas = (warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
@@ -670,7 +689,7 @@ gnmr_status gnmr_get_info(const gnmr_handle *h, gnmr_info *info)
     info->arena_elems_min = h->max_end;
     info->steps = h->steps;
     info->loop_shape = h->variant == gnmr::kVariantBulk ? GNMR_LOOP_LARGE_UNITS : GNMR_LOOP_SMALL_UNITS;
-    info->reserved = 0;
+    info->num_runs = h->num_runs;
     return GNMR_OK;
 }
 

@@ -12,9 +12,10 @@ namespace gnmr {
 
 // Launch shape of the step kernel: 512 threads = 16 warps per CTA.  Two
 // compiled variants of the streaming loop (gnmr_kernels.cu): kVariantSmall
-// (two resident CTAs per SM) for layouts of many small units, kVariantBulk
-// (one CTA per SM, deeper per-warp streams) for layouts whose mean unit holds
-// at least kBulkUnitBytes.
+// (two resident CTAs per SM, one planned run per warp) for layouts of many
+// small units, kVariantBulk (one CTA per SM, deeper per-warp streams, runs
+// taken from a shared counter) for layouts whose mean unit holds at least
+// kBulkUnitBytes.
 constexpr int kThreads = 512;
 constexpr int kWarpsPerCta = kThreads / 32;
 constexpr int kVariantSmall = 0;
@@ -28,6 +29,14 @@ constexpr int64_t kBulkUnitBytes = int64_t(1) << 20;
 constexpr int64_t kUnitCostBytes = 4096;
 constexpr int64_t kSplitBytes = 512;
 constexpr int64_t kMinRunBytes = 4096;   // one 4 KiB load round per warp: small problems spread over more SMs
+// Large-unit loop: the stream is cut into about kRunsPerWarp runs per warp of
+// kBulkRunMin..kBulkRunMax bytes each.  Each warp starts on its own run and
+// then takes the next untaken one, so warps that stream faster take more runs
+// and all finish together (static equal runs left the slowest warps ~8 % of
+// the step behind the median one).
+constexpr int64_t kRunsPerWarp = 16;
+constexpr int64_t kBulkRunMin = int64_t(64) << 10;
+constexpr int64_t kBulkRunMax = int64_t(256) << 10;
 
 // Persistent per-unit controller state (Algorithm 1 and 2), 40 bytes.
 struct UnitState {
@@ -78,7 +87,11 @@ struct Control {
     int64_t steps;        // completed steps (t of the last step)
     uint32_t n_hot;       // hot-list entries appended so far (may exceed the capacity)
     uint32_t hot_bin;     // lowest bin whose pool members go to the hot list this step
+    uint32_t pad[26];     // the run counters below on a 128-byte line of their own
+    uint32_t next_run;    // runs taken beyond the warps' first ones (large-unit loop)
+    uint32_t warps_done;  // warps that have taken their last run; both zero between launches
 };
+static_assert(offsetof(Control, next_run) == 128, "run counters on their own line");
 
 // Checkpoint blob: this header, then UnitState[num_units], then the GNMR ring
 // buffers double[num_units * window] (little-endian, as on the device).
@@ -97,9 +110,9 @@ struct StepParams {
     const int64_t *length;       // [S] segment lengths
     const int32_t *seg_unit;     // [S] unit of each segment (non-decreasing)
     const uint8_t *recoverable;  // [U]
-    const int64_t *run_seg;      // [W + 1] first segment of each warp's run
-    const int64_t *run_pos;      // [W + 1]
-    const int32_t *first_warp;   // [U]
+    const int64_t *run_seg;      // [R + 1] first segment of each run
+    const int64_t *run_pos;      // [R + 1]
+    const int32_t *first_run;    // [U] first run touching unit b
     const int32_t *num_parts;    // [U]
     const int64_t *part_base;    // [U] first partial slot of unit b
     double *partial;             // [num_partials]
@@ -124,11 +137,11 @@ struct StepParams {
     int32_t static_keep;                                  // ceil(static_fraction * |B_rec|)
     uint32_t hot_cap;                                     // min(U, kHotCapMax)
     int32_t num_units;
-    int32_t num_warps;
+    int32_t num_warps;           // warps with a first run: runs 0 .. num_warps - 1
     int32_t window;
     int32_t max_o;
     int32_t lock_len;
-    int32_t pad;
+    int32_t num_runs;            // R; runs num_warps .. R - 1 are taken dynamically
     int64_t warmup_steps;
     double alpha_init, alpha_main, beta_init, beta_main, eps;
     double alpha_override, beta_override;  // NaN = two-stage schedule
@@ -153,18 +166,20 @@ void record_thread_error(const char *why);
 
 // Host-side work partition (gnmr_plan.cpp).
 struct Plan {
-    int32_t num_warps = 0;
-    std::vector<int64_t> run_seg;     // [num_warps + 1]
-    std::vector<int64_t> run_pos;     // [num_warps + 1]
-    std::vector<int32_t> first_warp;  // [U]
+    int32_t num_runs = 0;
+    std::vector<int64_t> run_seg;     // [num_runs + 1]
+    std::vector<int64_t> run_pos;     // [num_runs + 1]
+    std::vector<int32_t> first_run;   // [U]
     std::vector<int32_t> num_parts;   // [U]
     std::vector<int64_t> part_base;   // [U]
     int64_t num_partials = 0;
 };
 
 // Segments must be grouped by unit (seg_unit non-decreasing, every unit
-// 0..num_units-1 present).  Returns false if the inputs are out of range.
+// 0..num_units-1 present).  Cuts the stream into at most max_runs runs, none
+// smaller than kMinRunBytes unless the whole problem is.  Returns false if
+// the inputs are out of range.
 bool plan_partition(int64_t num_segments, const int64_t *seg_lengths, const int32_t *seg_unit,
-                    int32_t num_units, int elem_bytes, int32_t max_warps, Plan &out);
+                    int32_t num_units, int elem_bytes, int32_t max_runs, Plan &out);
 
 }  // namespace gnmr

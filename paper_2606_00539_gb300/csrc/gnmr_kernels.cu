@@ -1,8 +1,13 @@
 // GNMR per-step monitor: one kernel launch per training step on sm_103a.
 //
-// Phase 1, every warp (the hot loop).  Each warp owns one contiguous run of
-// the segment stream planned by gnmr_plan.cpp (a unit is one or more
-// segments of the arena).  For every segment piece in its run it streams the
+// Phase 1, every warp (the hot loop).  The segment stream (a unit is one or
+// more segments of the arena) is cut by gnmr_plan.cpp into contiguous runs.
+// With the small-unit loop each warp owns one run.  With the large-unit loop
+// there are about 16 runs per warp: each warp starts on its own run and then
+// takes the next untaken one from a counter, so warps that stream faster take
+// more runs and all warps finish within about one run of each other (with one
+// run per warp, HBM's uneven service left the slowest warps ~8 % of the step
+// behind the median).  For every segment piece in a run the warp streams the
 // gradient with 16-byte read-only loads (8 or 16 in flight per lane, by the
 // loop shape), squares in fp32, sums blocks of 16 iterations in fp32 and the
 // blocks as float pairs (error-free TwoSum), and all-reduces the lanes' totals
@@ -10,11 +15,11 @@
 // n_b = ||g_b||_2 (Sec. 2, Eq. local_gradient).  No shared memory, no block
 // barrier on this path.  (The streaming reduction lives in gnmr_stream.cuh.)
 //
-// Phase 2, the warp that completes unit b.  A unit split over several warps
-// collects their partial sums through fixed slots and a per-unit ticket; the
-// warp that takes the last ticket sums the slots in slot order (so the result
-// does not depend on timing); a unit of two parts trades its partial in one
-// atomic exchange.  Completed units queue up in the warp's lanes and run the
+// Phase 2, the warp that completes unit b.  A unit split over several runs
+// collects their partial sums through fixed slots (one per run, whichever
+// warp streams it) and a per-unit ticket; the warp that takes the last ticket
+// sums the slots in slot order (so the result does not depend on timing); a
+// unit of two parts trades its partial in one atomic exchange.  Completed units queue up in the warp's lanes and run the
 // unit epilogue 32 at a time, one unit per lane: Algorithm 1 (GNMR,
 // Delta-GNMR, incremental mean, window queue), the combined risk
 // R = max{GNMR/alpha_t, Delta-GNMR/beta_t} and the candidate test
@@ -30,8 +35,8 @@
 // (R descending, unit index ascending) in shared memory.  Then the lock
 // bookkeeping of Algorithm 2 for the selected units, the counts, and the
 // reset of the counters for the next launch.  No CTA ever waits for another:
-// the tickets decide who continues, so the kernel cannot hang whatever the
-// grid size or residency.
+// the tickets and the run counter decide who continues, so the kernel cannot
+// hang whatever the grid size or residency.
 //
 // The same kernel also runs either half of a sharded step: phase 1 alone
 // (per-unit sums of squares of a shard) or phases 2-3 alone on sums that the
@@ -58,11 +63,13 @@ template <> struct Shape<kVariantSmall> {
     static constexpr int kUnroll = 8;
     static constexpr int kMinCtas = 2;
     static constexpr int64_t kPieceBytes = 0;         // each segment of a run in one call
+    static constexpr bool kDynamic = false;           // one planned run per warp
 };
 template <> struct Shape<kVariantBulk> {
     static constexpr int kUnroll = 16;
     static constexpr int kMinCtas = 1;
     static constexpr int64_t kPieceBytes = 256 << 10;
+    static constexpr bool kDynamic = true;            // further runs taken from a counter
 };
 
 __device__ __forceinline__ double pick_threshold(double override_value, int64_t t, int64_t warmup,
@@ -255,7 +262,7 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
 // the first warp finds the slot empty and leaves its partial there, the
 // second takes it, adds it to its own (IEEE addition is commutative, so the
 // bits are those of the slot-order sum) and empties the slot again.
-__device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, int32_t parts, int warp,
+__device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, int32_t parts, int32_t run,
                                               double &s, int lane)
 {
     const int64_t base = p.part_base[b];
@@ -276,7 +283,7 @@ __device__ __forceinline__ bool combine_parts(const StepParams &p, int32_t b, in
     }
     uint32_t last = 0;
     if (lane == 0) {
-        __stcg(&p.partial[base + (warp - p.first_warp[b])], s);
+        __stcg(&p.partial[base + (run - p.first_run[b])], s);
         last = ticket_acq_rel(&p.unit_ticket[b]) == static_cast<uint32_t>(parts - 1);
     }
     last = __shfl_sync(kFull, last, 0);
@@ -914,23 +921,16 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
         const int64_t t = __ldcg(&p.ctl->steps) + 1;
         const double alpha = pick_threshold(p.alpha_override, t, p.warmup_steps, p.alpha_init, p.alpha_main);
         const double beta = pick_threshold(p.beta_override, t, p.warmup_steps, p.beta_init, p.beta_main);
-        int64_t g = p.run_seg[warp];
-        int64_t pos = p.run_pos[warp];
-        const int64_t g_end = p.run_seg[warp + 1];
-        const int64_t pos_end = p.run_pos[warp + 1];
         const char *arena = static_cast<const char *>(p.arena);
         // Units this warp completes wait here, lane j holding the j-th, and run
         // their epilogues 32 at a time.
         int32_t pend_b = 0;
         double pend_s = 0.0;
         int npend = 0;
-        // Segments of one unit are consecutive: their sums add up in segment
-        // order until the unit changes.
-        int32_t cur = -1;
-        double cur_s = 0.0;
+        int32_t run = warp;                              // every warp starts on its own run
         auto complete = [&](int32_t b, double s) {
             const int32_t parts = p.num_parts[b];
-            if (parts == 1 || combine_parts(p, b, parts, warp, s, lane)) {
+            if (parts == 1 || combine_parts(p, b, parts, run, s, lane)) {
                 if (MODE == kStepPartials) {
                     if (lane == 0)
                         p.out_sumsq[b] = s;
@@ -946,44 +946,71 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
                 }
             }
         };
-        while (g < g_end || (g == g_end && pos < pos_end)) {
-            const int32_t b = p.seg_unit[g];
-            const int64_t len = p.length[g];
-            int64_t stop = (g == g_end) ? pos_end : len;
-            stop = stop < len ? stop : len;
-            const int64_t n = stop > pos ? stop - pos : 0;
-            const char *seg = arena + (p.offset[g] + pos) * kEB;
-            double s;
-            if (Shape<V>::kPieceBytes > 0 && n > Shape<V>::kPieceBytes / kEB) {
-                constexpr int64_t kPiece = Shape<V>::kPieceBytes > 0 ? Shape<V>::kPieceBytes / kEB : 1;
-                s = 0.0;
-                for (int64_t q = 0; q < n; q += kPiece) {     // the pieces' sums, in order
-                    const int64_t m = n - q < kPiece ? n - q : kPiece;
+        for (;;) {
+            // Large-unit loop: the index of the warp's next run is taken now, so
+            // the atomic's round trip hides under this run's stream.
+            uint32_t next = 0;
+            if (Shape<V>::kDynamic && lane == 0)
+                next = atomicAdd(&p.ctl->next_run, 1u);
+            int64_t g = p.run_seg[run];
+            int64_t pos = p.run_pos[run];
+            const int64_t g_end = p.run_seg[run + 1];
+            const int64_t pos_end = p.run_pos[run + 1];
+            // Segments of one unit are consecutive: their sums add up in segment
+            // order until the unit changes.
+            int32_t cur = -1;
+            double cur_s = 0.0;
+            while (g < g_end || (g == g_end && pos < pos_end)) {
+                const int32_t b = p.seg_unit[g];
+                const int64_t len = p.length[g];
+                int64_t stop = (g == g_end) ? pos_end : len;
+                stop = stop < len ? stop : len;
+                const int64_t n = stop > pos ? stop - pos : 0;
+                const char *seg = arena + (p.offset[g] + pos) * kEB;
+                double s;
+                if (Shape<V>::kPieceBytes > 0 && n > Shape<V>::kPieceBytes / kEB) {
+                    constexpr int64_t kPiece = Shape<V>::kPieceBytes > 0 ? Shape<V>::kPieceBytes / kEB : 1;
+                    s = 0.0;
+                    for (int64_t q = 0; q < n; q += kPiece) {     // the pieces' sums, in order
+                        const int64_t m = n - q < kPiece ? n - q : kPiece;
+                        bool suspect;
+                        double x = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg + q * kEB, m, lane, suspect);
+                        if (suspect)
+                            x = warp_segment_sumsq_f64<DT>(seg + q * kEB, m, lane);
+                        s += x;
+                    }
+                } else {
                     bool suspect;
-                    double x = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg + q * kEB, m, lane, suspect);
+                    s = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg, n, lane, suspect);
                     if (suspect)
-                        x = warp_segment_sumsq_f64<DT>(seg + q * kEB, m, lane);
-                    s += x;
+                        s = warp_segment_sumsq_f64<DT>(seg, n, lane);
                 }
-            } else {
-                bool suspect;
-                s = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg, n, lane, suspect);
-                if (suspect)
-                    s = warp_segment_sumsq_f64<DT>(seg, n, lane);
+                if (b != cur) {
+                    if (cur >= 0)
+                        complete(cur, cur_s);
+                    cur = b;
+                    cur_s = s;
+                } else {
+                    cur_s += s;
+                }
+                ++g;
+                pos = 0;
             }
-            if (b != cur) {
-                if (cur >= 0)
-                    complete(cur, cur_s);
-                cur = b;
-                cur_s = s;
-            } else {
-                cur_s += s;
-            }
-            ++g;
-            pos = 0;
+            if (cur >= 0)
+                complete(cur, cur_s);
+            if (!Shape<V>::kDynamic)
+                break;
+            run = p.num_warps + static_cast<int32_t>(__shfl_sync(kFull, next, 0));
+            if (run >= p.num_runs)
+                break;
         }
-        if (cur >= 0)
-            complete(cur, cur_s);
+        // The last warp to take its last index resets the counters for the
+        // next launch (which starts only after this grid has completed).
+        if (Shape<V>::kDynamic && lane == 0 &&
+            ticket_acq_rel(&p.ctl->warps_done) == static_cast<uint32_t>(p.num_warps - 1)) {
+            p.ctl->next_run = 0;
+            p.ctl->warps_done = 0;
+        }
         if (MODE != kStepPartials && npend > 0)
             unit_epilogue(p, lane < npend, pend_b, pend_s, alpha, beta, t);
     }

@@ -6,18 +6,20 @@
 // segment of L elements contributes max(L, 1) points (a unit with no element
 // still needs one warp to run its Algorithm 1 update).  A unit costs
 // kUnitCostBytes plus the bytes of its segments.  The stream is cut into runs
-// of about equal cost, one run per warp, so skewed sizes (a 256-element unit
-// next to a 70M-element one) balance across the grid: large segments are
-// split over many warps, small ones are packed many to a warp.
+// of about equal cost, so skewed sizes (a 256-element unit next to a
+// 70M-element one) balance across the grid: large segments are split over
+// many runs, small ones are packed many to a run.  The small-unit loop gives
+// every warp one run; the large-unit loop plans several runs per warp, which
+// the warps take in turn.
 //
 // Cuts inside a segment fall on multiples of kSplitBytes from its start, so
 // the body of every piece keeps the segment's 16-byte alignment.  Runs are
 // strictly increasing and never empty, and a unit's segments are contiguous in
-// the stream, so the warps that touch a unit are a contiguous range
-// first_warp[b] .. first_warp[b] + num_parts[b] - 1; the kernel stores the
-// partial sum of warp w for unit b in slot part_base[b] + (w - first_warp[b]),
-// so the reduction order of a unit is fixed by the plan and results are
-// bitwise reproducible run to run.
+// the stream, so the runs that touch a unit are a contiguous range
+// first_run[b] .. first_run[b] + num_parts[b] - 1; the kernel stores the
+// partial sum of run r for unit b in slot part_base[b] + (r - first_run[b]),
+// so the reduction order of a unit is fixed by the plan (whichever warp
+// streams a run) and results are bitwise reproducible run to run.
 #include <algorithm>
 #include <cstdint>
 #include <vector>
@@ -37,10 +39,10 @@ struct Point {
 }  // namespace
 
 bool plan_partition(int64_t num_segments, const int64_t *seg_lengths, const int32_t *seg_unit,
-                    int32_t num_units, int elem_bytes, int32_t max_warps, Plan &out)
+                    int32_t num_units, int elem_bytes, int32_t max_runs, Plan &out)
 {
     if (num_segments < 1 || num_units < 1 || !seg_lengths || !seg_unit ||
-        (elem_bytes != 2 && elem_bytes != 4) || max_warps < 1)
+        (elem_bytes != 2 && elem_bytes != 4) || max_runs < 1)
         return false;
     const int64_t S = num_segments, U = num_units;
     // segments must be grouped by unit, every unit present
@@ -66,7 +68,7 @@ bool plan_partition(int64_t num_segments, const int64_t *seg_lengths, const int3
     }
     const int64_t total = cstart[S];
     const int64_t want = (total + kMinRunBytes - 1) / kMinRunBytes;
-    const int64_t W = std::max<int64_t>(1, std::min<int64_t>(want, max_warps));
+    const int64_t W = std::max<int64_t>(1, std::min<int64_t>(want, max_runs));
     const int64_t align = std::max<int64_t>(1, kSplitBytes / elem_bytes);
 
     std::vector<Point> cuts;
@@ -93,14 +95,14 @@ bool plan_partition(int64_t num_segments, const int64_t *seg_lengths, const int3
     cuts.push_back(end);
 
     const int64_t nw = (int64_t)cuts.size() - 1;
-    out.num_warps = (int32_t)nw;
+    out.num_runs = (int32_t)nw;
     out.run_seg.resize(nw + 1);
     out.run_pos.resize(nw + 1);
     for (int64_t w = 0; w <= nw; ++w) {
         out.run_seg[w] = cuts[w].seg;
         out.run_pos[w] = cuts[w].pos;
     }
-    out.first_warp.assign(U, -1);
+    out.first_run.assign(U, -1);
     out.num_parts.assign(U, 0);
     for (int64_t w = 0; w < nw; ++w) {
         const int64_t g0 = cuts[w].seg;
@@ -111,8 +113,8 @@ bool plan_partition(int64_t num_segments, const int64_t *seg_lengths, const int3
             if (b == prev_unit)
                 continue;
             prev_unit = b;
-            if (out.first_warp[b] < 0)
-                out.first_warp[b] = (int32_t)w;
+            if (out.first_run[b] < 0)
+                out.first_run[b] = (int32_t)w;
             out.num_parts[b] += 1;
         }
     }

@@ -69,7 +69,7 @@ int main(void) {
   F(gnmr_info, num_units) F(gnmr_info, dtype) F(gnmr_info, device) F(gnmr_info, num_ctas)
   F(gnmr_info, threads_per_cta) F(gnmr_info, num_warps) F(gnmr_info, num_partials)
   F(gnmr_info, device_bytes) F(gnmr_info, arena_elems_min) F(gnmr_info, steps)
-  F(gnmr_info, loop_shape) F(gnmr_info, reserved)
+  F(gnmr_info, loop_shape) F(gnmr_info, num_runs)
   return 0;
 }
 """

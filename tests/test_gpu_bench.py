@@ -46,6 +46,7 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
                     "l2_flushed_us_mean", "l2_cleaned_us_mean"):
             assert rec[key] > 0, key
         assert rec["kernel_us_min"] <= rec["kernel_us_mean"] <= rec["kernel_us_max"]
+        assert rec["kernel_us_min"] <= rec["kernel_us_median"] <= rec["kernel_us_max"]
         assert rec["frac"] == pytest.approx(rec["gbs"] / per["peak_gbs"], abs=1e-3)
         assert 0 <= rec["selected_mean"] <= rec["max_o"] and rec["candidates_max"] >= 0
         assert {"sm_mhz", "reasons"} <= set(rec["clocks"])

@@ -115,6 +115,23 @@ def test_loop_shape_follows_the_mean_unit_size(cuda_device):
                 assert mon.info()["loop_shape"] == code
 
 
+def test_large_unit_loop_takes_runs_dynamically(cuda_device):
+    """The large-unit loop plans about 16 runs per warp (64-256 KiB each), and
+    the small-unit loop one run per warp."""
+    for config in ("llama2-1.3b", "llama2-13b", "moe", "tiny", "aq-stress"):
+        w = workloads.make(config)
+        with _monitor(w) as mon:
+            info = mon.info()
+            cost = w.grad_bytes + 4096 * w.num_units
+            if info["loop_shape"] == N.GNMR_LOOP_LARGE_UNITS:
+                assert info["num_runs"] > 4 * info["num_warps"], config
+                assert (64 << 10) * 0.99 <= cost / info["num_runs"] <= (256 << 10) * 1.01, config
+                assert info["num_partials"] >= info["num_runs"]
+            else:
+                assert info["num_runs"] == info["num_warps"], config
+            assert info["num_ctas"] * info["threads_per_cta"] // 32 >= info["num_warps"]
+
+
 def test_segments_in_any_order_and_units_without_segments(cuda_device):
     import torch
     rng = np.random.default_rng(21)

@@ -22,7 +22,8 @@ def _monitor(w, off=None, ln=None):
 
 
 @pytest.mark.parametrize("config,shrink,world", [("llama2-13b", 16, 2), ("aq-stress", 8, 3),
-                                                 ("moe", 32, 2)])
+                                                 ("moe", 32, 2),
+                                                 ("llama2-1.3b", 2, 2)])   # shards with more runs than warps
 def test_sharded_step_matches_oracle(config, shrink, world, cuda_device):
     """World-size emulation on one GPU: the ranks' halves run one after the
     other (no kernel waits for another); the all-reduce is a device add."""
