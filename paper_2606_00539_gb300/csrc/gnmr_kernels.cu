@@ -7,7 +7,7 @@
 // takes the next untaken one from a counter, so warps that stream faster take
 // more runs and all warps finish within about one run of each other (with one
 // run per warp, HBM's uneven service left the slowest warps ~8 % of the step
-// behind the median).  For every segment piece in a run the warp streams the
+// behind the median).  For every segment (or part of one) in a run the warp streams the
 // gradient with 16-byte read-only loads (8 or 16 in flight per lane, by the
 // loop shape), squares in fp32, sums blocks of 16 iterations in fp32 and the
 // blocks as float pairs (error-free TwoSum), and all-reduces the lanes' totals
@@ -55,20 +55,17 @@ namespace {
 // Two compiled shapes of the streaming loop, chosen per handle from the mean
 // unit size (both measured on GB300): many small units run best with 8
 // 16-byte loads in flight per lane and two CTAs per SM; large units with 16
-// loads per lane and one CTA per SM (fewer, deeper streams), a warp's long
-// run reduced 256 KiB at a time (measured: 1.6 % faster on 13B and MoE
-// layouts than one call per run).
+// loads per lane and one CTA per SM (fewer, deeper streams) and runs of at
+// most 256 KiB taken dynamically.
 template <int V> struct Shape;
 template <> struct Shape<kVariantSmall> {
     static constexpr int kUnroll = 8;
     static constexpr int kMinCtas = 2;
-    static constexpr int64_t kPieceBytes = 0;         // each segment of a run in one call
     static constexpr bool kDynamic = false;           // one planned run per warp
 };
 template <> struct Shape<kVariantBulk> {
     static constexpr int kUnroll = 16;
     static constexpr int kMinCtas = 1;
-    static constexpr int64_t kPieceBytes = 256 << 10;
     static constexpr bool kDynamic = true;            // further runs taken from a counter
 };
 
@@ -967,24 +964,10 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
                 stop = stop < len ? stop : len;
                 const int64_t n = stop > pos ? stop - pos : 0;
                 const char *seg = arena + (p.offset[g] + pos) * kEB;
-                double s;
-                if (Shape<V>::kPieceBytes > 0 && n > Shape<V>::kPieceBytes / kEB) {
-                    constexpr int64_t kPiece = Shape<V>::kPieceBytes > 0 ? Shape<V>::kPieceBytes / kEB : 1;
-                    s = 0.0;
-                    for (int64_t q = 0; q < n; q += kPiece) {     // the pieces' sums, in order
-                        const int64_t m = n - q < kPiece ? n - q : kPiece;
-                        bool suspect;
-                        double x = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg + q * kEB, m, lane, suspect);
-                        if (suspect)
-                            x = warp_segment_sumsq_f64<DT>(seg + q * kEB, m, lane);
-                        s += x;
-                    }
-                } else {
-                    bool suspect;
-                    s = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg, n, lane, suspect);
-                    if (suspect)
-                        s = warp_segment_sumsq_f64<DT>(seg, n, lane);
-                }
+                bool suspect;
+                double s = warp_segment_sumsq<DT, Shape<V>::kUnroll>(seg, n, lane, suspect);
+                if (suspect)
+                    s = warp_segment_sumsq_f64<DT>(seg, n, lane);
                 if (b != cur) {
                     if (cur >= 0)
                         complete(cur, cur_s);

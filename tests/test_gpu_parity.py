@@ -289,6 +289,46 @@ def test_unaligned_overlapping_and_empty_units(dtype, shape, cuda_device):
                      dict(window=2, max_o=3, lock_len=2, alpha=(1.2, 1.2), beta=(1.2, 1.2)), 6)
 
 
+def test_dynamic_runs_with_unaligned_special_and_empty_units(cuda_device):
+    """The large-unit loop with many more runs than warps (a 400 MB bf16 arena,
+    ~6,000 runs of 64 KiB): units at odd offsets, overlapping units, empty and
+    one-element units, a unit over the whole arena, a unit that turns NaN and
+    one whose squares overflow fp32 (the exact path) at some steps."""
+    import torch
+    n = 200_000_003
+    rng = np.random.default_rng(31)
+    off = [0, 1, 3, 7, 11, 150_000_001, 5, 0, 99_999_999, 123]
+    ln = [1, 0, 40_000_001, 13, 60_000_000, 49_999_999, 20_000_003, n, 2, 3_000_000]
+    for _ in range(30):                                   # assorted units in [0, 100M), some overlapping
+        o = int(rng.integers(0, 88_000_000))
+        off.append(o)
+        ln.append(int(rng.integers(100_000, 12_000_000)))
+    off = np.array(off, np.int64)
+    ln = np.array(ln, np.int64)
+    gen = torch.Generator(device=cuda_device)
+    gen.manual_seed(5)
+    base = torch.randn(n, generator=gen, device=cuda_device)
+    dev = torch.empty(n, dtype=torch.bfloat16, device=cuda_device)
+
+    def make_step(t, attempt, bad):
+        gen.manual_seed(7000 + 100 * t + attempt)
+        noise = torch.randn(n, generator=gen, device=cuda_device)
+        x = base * (1.0 + 0.3 * noise)
+        if t == 2:
+            x[199_999_990] = float("nan")                     # units 5 and 7 only
+        if t == 4:
+            x[11 + 1_000:11 + 2_000] = 3e25                    # unit 4: fp32 squares overflow
+        dev.copy_(x.to(torch.bfloat16))
+
+    mon_kw = dict(dtype="bf16", window=3, max_o=4, lock_len=2, alpha=1.2, beta=1.2, loop_shape="large")
+    with Monitor(off, ln, device=0, **mon_kw) as mon:
+        info = mon.info()
+        assert info["loop_shape"] == N.GNMR_LOOP_LARGE_UNITS
+        assert info["num_runs"] > 2 * info["num_warps"]
+    _parity_on_norms(off, ln, dev, make_step, mon_kw,
+                     dict(window=3, max_o=4, lock_len=2, alpha=(1.2, 1.2), beta=(1.2, 1.2)), 7)
+
+
 def _per_unit_levels_arena(rng, ln, steps, sigma, device, zero_units=()):
     """Packed fp32 units; step t of unit u is base * level[t, u].  Returns
     (offsets, arena, make_step) with per-unit margin repair."""
