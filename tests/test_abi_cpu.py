@@ -235,6 +235,28 @@ def test_partition_on_workloads(lib, config):
         assert W == 152 * 2 * 16        # big workloads use the whole grid
 
 
+def _large_unit_runs(grad_bytes, num_units, grid_warps=152 * 16):
+    """The run count gnmr_create plans for the large-unit loop: about 16 runs
+    per warp of 64-256 KiB of cost each, never fewer than one per warp."""
+    cost = grad_bytes + UNIT_COST * num_units
+    run = min(max(cost // (grid_warps * 16), 64 << 10), 256 << 10)
+    return max(grid_warps, -(-cost // run)), run
+
+
+@pytest.mark.parametrize("config", [2, 3, 4])
+def test_partition_of_dynamic_runs(lib, config):
+    """The many-runs plans of the large-unit loop (37K-121K runs): the same
+    invariants, and every run within a granule and a unit's fixed cost of
+    the run size."""
+    import workloads
+    w = workloads.make(config)
+    dt = N.GNMR_DTYPE_BF16 if w.dtype == "bf16" else N.GNMR_DTYPE_F32
+    R, run = _large_unit_runs(w.grad_bytes, w.num_units)
+    assert R > 8 * 152 * 16
+    W = _check_plan(w.lengths, dt, int(R))
+    assert R - 1 <= W <= R
+
+
 def test_partition_rejects_bad_input(lib):
     with pytest.raises(N.GnmrError):
         N.gnmr_plan_partition(np.array([5, -1], np.int64), N.GNMR_DTYPE_F32, 4)
