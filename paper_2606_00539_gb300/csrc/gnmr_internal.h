@@ -89,7 +89,8 @@ struct Control {
     uint32_t hot_bin;     // lowest bin whose pool members go to the hot list this step
     uint32_t pad[26];     // the run counters below on a 128-byte line of their own
     uint32_t next_run;    // runs taken beyond the warps' first ones (large-unit loop)
-    uint32_t warps_done;  // warps that have taken their last run; both zero between launches
+    uint32_t warps_done;  // partial-sums half: warps that have taken their last run
+                          // (both zero between launches)
 };
 static_assert(offsetof(Control, next_run) == 128, "run counters on their own line");
 

@@ -138,6 +138,9 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
     bool cand = false;
     double r = 0.0;
     uint32_t cand_lock = 0;
+    // read now, used after the risk: the step's hot-list bin (only the
+    // selection, after every CTA, rewrites it)
+    const uint32_t hot_bin = __ldcg(&p.ctl->hot_bin);
     if (active) {
         const double n = sqrt(sumsq);
         const int w = p.window;
@@ -147,16 +150,20 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
         asm volatile("prefetch.global.L1 [%0];" ::"l"(Q));
         asm volatile("prefetch.global.L1 [%0];" ::"l"(Q + (w - 1)));
         UnitState s = p.state[b];
+        const bool rec = p.recoverable[b] != 0;
+        // The risk first (its chain of dependent divisions decides the
+        // epilogue's latency), the state update after it.
         double g, d;
         if (!isfinite(n)) {
             // Non-finite gradient: maximal risk, no change to A_b, Q_b, k_b.
             g = CUDART_INF;
             d = CUDART_INF;
         } else {
-            g = (s.count == 0 || s.mean == 0.0) ? 1.0 : n / (s.mean + p.eps);
-            if (s.fill == w) {
-                // mean of the window, summed oldest to newest; loads issued 8 at a time
-                double q = 0.0;
+            // mean of the window, summed oldest to newest; its loads are issued
+            // as soon as the state's head is known, before the division for g
+            const bool full = s.fill == w;
+            double q = 0.0;
+            if (full) {
                 int idx = s.head, k = 0;
                 for (; k + 8 <= w; k += 8) {
                     double v[8];
@@ -174,11 +181,18 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
                     q += Q[idx];
                     idx = (idx + 1 == w) ? 0 : idx + 1;
                 }
+            }
+            g = (s.count == 0 || s.mean == 0.0) ? 1.0 : n / (s.mean + p.eps);
+            if (full) {
                 const double den = q / static_cast<double>(w) + p.eps;
                 d = (den == 0.0) ? (g > 0.0 ? CUDART_INF : 1.0) : g / den;
             } else {
                 d = 1.0;
             }
+        }
+        const double x = g / alpha, y = d / beta;
+        r = x > y ? x : y;
+        if (isfinite(n)) {
             s.count += 1;
             s.mean = s.mean + (n - s.mean) / static_cast<double>(s.count);
             if (s.fill < w) {                        // still filling: head stays 0
@@ -193,15 +207,12 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
             p.state[b].fill = s.fill;
             p.state[b].head = s.head;
         }
-        const double x = g / alpha, y = d / beta;
-        r = x > y ? x : y;
 
         if (p.out_norm) p.out_norm[b] = n;
         if (p.out_gnmr) p.out_gnmr[b] = g;
         if (p.out_dgnmr) p.out_dgnmr[b] = d;
         if (p.out_risk) p.out_risk[b] = r;
 
-        const bool rec = p.recoverable[b] != 0;
         const bool stat = p.policy == 2;
         if (stat && t <= p.static_warmup && rec)
             p.state[b].gsum = s.gsum + g;
@@ -246,7 +257,7 @@ __device__ void unit_epilogue(const StepParams &p, bool active, int32_t b, doubl
     if (cand && !retained) {
         const uint32_t bin = risk_bin(risk_key(r));
         atomicAdd(&p.risk_hist[bin], 1u);
-        hot = bin >= __ldcg(&p.ctl->hot_bin);
+        hot = bin >= hot_bin;
     }
     warp_append(p.cand, &p.ctl->n_cand, static_cast<uint32_t>(p.num_units), cand, r, b, cand_lock);
     warp_append(p.hot, &p.ctl->n_hot, p.hot_cap, hot, r, b, cand_lock);
@@ -871,6 +882,7 @@ __device__ void select_and_commit(const StepParams &p, int64_t t, uint32_t *hist
     }
     __syncthreads();
     if (threadIdx.x == 0) {
+        p.ctl->next_run = 0;                         // every CTA, so every warp, is done
         p.ctl->n_cand = 0;
         p.ctl->n_hot = 0;
         if (next_hot <= kNoHot)
@@ -987,9 +999,11 @@ gnmr_step_kernel(const __grid_constant__ StepParams p)
             if (run >= p.num_runs)
                 break;
         }
-        // The last warp to take its last index resets the counters for the
-        // next launch (which starts only after this grid has completed).
-        if (Shape<V>::kDynamic && lane == 0 &&
+        // The run counter is reset for the next launch (which starts only
+        // after this grid has completed) by the selecting CTA, after every
+        // warp has drawn its last index.  The partial-sums half has no
+        // selecting CTA: there the last warp to draw past the end resets it.
+        if (Shape<V>::kDynamic && MODE == kStepPartials && lane == 0 &&
             ticket_acq_rel(&p.ctl->warps_done) == static_cast<uint32_t>(p.num_warps - 1)) {
             p.ctl->next_run = 0;
             p.ctl->warps_done = 0;
