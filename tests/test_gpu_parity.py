@@ -617,12 +617,15 @@ def test_mask_only_and_side_stream(cuda_device):
         b.close()
 
 
-def test_cuda_graph_replay_advances_steps(cuda_device):
+@pytest.mark.parametrize("config,shrink,steps", [("tiny", 4, 30),
+                                                 ("llama2-1.3b", 2, 10)])   # dynamic runs
+def test_cuda_graph_replay_advances_steps(config, shrink, steps, cuda_device):
     """The step is one launch with no host synchronisation: captured once in a
     CUDA graph and replayed, it matches the oracle step by step (the step
-    counter and thresholds live on the device)."""
+    counter, the thresholds and the large-unit loop's run counter live on the
+    device and are reset by the kernel)."""
     import torch
-    w = workloads.make("tiny", seed=9, steps=30, shrink=4)
+    w = workloads.make(config, seed=9, steps=steps, shrink=shrink)
     tr = TD.LockstepTrace(w, "cuda:0", _monitor)
     mask = torch.empty(w.num_units, dtype=torch.uint8, device=cuda_device)
     s = torch.cuda.Stream(cuda_device)
