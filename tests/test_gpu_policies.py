@@ -36,7 +36,8 @@ def _run(w, policy, steps=None, check=None):
 
 
 @pytest.mark.parametrize("config,shrink,steps", [("tiny", 2, 80), ("aq-stress", 4, 20),
-                                                 ("llama2-13b", 32, None)])
+                                                 ("llama2-13b", 32, None),
+                                                 ("llama2-1.3b", 2, 30)])   # dynamic runs
 def test_admission_cap_parity(config, shrink, steps, cuda_device):
     w = workloads.make(config, shrink=shrink, steps=steps)
     seen = {"over": False}
