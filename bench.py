@@ -53,6 +53,11 @@ def parse_args(argv=None):
     p.add_argument("--shrink", type=int, default=1,
                    help="divide matrix dims (small case for profiler captures)")
     p.add_argument("--arenas", type=int, default=2, help="distinct step arenas cycled")
+    p.add_argument("--trace-steps", action="store_true",
+                   help="time the workload's own consecutive trace steps: a fresh monitor runs the "
+                        "steps before them untimed, every warm-up and timed step has its own arena "
+                        "(they must all fit in device memory), and one untimed pass over those "
+                        "arenas from the same state precedes the warm-up")
     p.add_argument("--e2e-steps", type=int, default=3)
     p.add_argument("--flush-l2", action="store_true",
                    help="write 512 MB before every timed step (outside its events)")
@@ -264,7 +269,9 @@ def workload_config(w, args, n_arenas: int, world: int) -> dict:
     return {"workload": f"{w.name} ({w.num_units} units, {w.num_segments} tensors, "
                         f"{w.grad_elems} {w.dtype} "
                         f"elements{'' if args.shrink == 1 else f', dims / {args.shrink}'})",
-            "bytes_per_step": w.grad_bytes, "arenas_cycled": n_arenas,
+            "bytes_per_step": w.grad_bytes,
+            "arenas_cycled": args.warmup + args.steps if getattr(args, "trace_steps", False) else n_arenas,
+            **({"trace_steps": list(trace_span(w, args))} if getattr(args, "trace_steps", False) else {}),
             "l2": ("L2 flushed before every step (512 MB write)" if getattr(args, "flush_l2", False)
                    else "inputs larger than L2 (no flush)" if w.grad_bytes > 2 * L2_BYTES
                    else "inputs fit in L2 (hot)"),
@@ -430,6 +437,12 @@ def trigger_sparsity(w, filler, arena, dev) -> dict:
 # ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
+
+def trace_span(w, args):
+    """(first, last) trace step timed by --trace-steps (1-based)."""
+    t0, k = trace_window(w.steps, args.steps, args.warmup)
+    return t0, t0 + k - 1
+
 
 def trace_window(trace_steps: int, k: int, w: int):
     """(first timed trace step, 1-based; number of timed steps): K steps in
@@ -676,22 +689,52 @@ def run_gnmr(args):
 
     w = workloads.make(args.workload, shrink=args.shrink, seed=rank, group=args.group)
     filler = workloads.Filler(w, dev)
-    n_arenas = max(1, args.arenas)
-    arenas = []
-    for i in range(n_arenas):
-        # steps from the middle of the trace: spikes, ramps and locks are live
-        a = filler.new_arena()
-        filler.fill(a, (w.steps // 2 + i) % w.steps)
-        arenas.append(a)
     mon = Monitor(w.offsets, w.lengths, device=local_rank, **w.monitor_kwargs())
     info = mon.info()
     stats = mon.new_stats()
     mask = torch.empty(w.num_units, dtype=torch.uint8, device=dev)
     stream = torch.cuda.Stream(dev)
+    arenas = []
+    if args.trace_steps:
+        # the trace's own steps: 1..first-1 untimed on one arena, then one
+        # arena per warm-up and timed step
+        t0, t1 = trace_span(w, args)
+        if t1 - t0 + 1 != args.steps:
+            raise SystemExit(f"--trace-steps: {w.name}'s trace has {w.steps} steps, too few for "
+                             f"{args.warmup} + {args.steps}")
+        first = t0 - args.warmup
+        need = (args.warmup + args.steps) * w.arena_elems * w.elem_bytes
+        if need > 0.8 * torch.cuda.mem_get_info(dev)[0]:
+            raise SystemExit(f"--trace-steps: {need / 1e9:.1f} GB of arenas do not fit on the device")
+        with torch.cuda.stream(stream):
+            scratch = filler.new_arena()
+            for i in range(first - 1):
+                filler.fill(scratch, i)
+                mon.step(scratch, mask=mask, stats=stats, stream=stream)
+            del scratch
+            for i in range(args.warmup + args.steps):
+                a = filler.new_arena()
+                filler.fill(a, first - 1 + i)
+                arenas.append(a)
+    else:
+        for i in range(max(1, args.arenas)):
+            # steps from the middle of the trace: spikes, ramps and locks are live
+            a = filler.new_arena()
+            filler.fill(a, (w.steps // 2 + i) % w.steps)
+            arenas.append(a)
+    n_arenas = len(arenas)
     torch.cuda.synchronize(dev)
 
     # one prepared gnmr_step call per arena: a step costs one C call on the host
     calls = [mon.prepare_step(a, mask=mask, stats=stats, stream=stream) for a in arenas]
+    if args.trace_steps:
+        # one untimed pass over every arena first, from the same controller
+        # state: the first read of a freshly generated arena runs up to ~10 %
+        # slower (measured), which no later read shows
+        blob = mon.get_state(stream)
+        for c in calls:
+            c()
+        mon.set_state(blob, stream)
     for i in range(args.warmup):
         calls[i % n_arenas]()
     stream.synchronize()
@@ -703,9 +746,13 @@ def run_gnmr(args):
         with torch.cuda.graph(graph, stream=stream):
             for i in range(args.steps):
                 calls[(args.warmup + i) % n_arenas]()
+        blob = mon.get_state(stream) if args.trace_steps else None
         with torch.cuda.stream(stream):
             graph.replay()                # untimed: the first replay uploads the graph
         torch.cuda.synchronize(dev)
+        if blob is not None:
+            mon.set_state(blob, stream)   # the timed replay runs the same trace steps again
+            torch.cuda.synchronize(dev)
 
     sampler = ClockSampler(local_rank)
     time.sleep(0.3)                       # let nvidia-smi start sampling

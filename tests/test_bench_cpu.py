@@ -85,6 +85,19 @@ def test_trace_window_is_inside_the_trace_after_the_warmup():
     assert bench.trace_window(50, 20, 5) == (16, 20)          # centred: steps 16..35
 
 
+def test_trace_steps_config_names_the_timed_trace_steps():
+    """--trace-steps times consecutive trace steps after the warm-up steps,
+    each with its own arena, and the config says which."""
+    import workloads
+    w = workloads.make("aq-stress")
+    args = bench.parse_args(["--workload", "aq-stress", "--trace-steps", "--steps", "20", "--warmup", "5"])
+    cfg = bench.workload_config(w, args, 0, 1)
+    assert cfg["trace_steps"] == [16, 35] and cfg["arenas_cycled"] == 25
+    assert bench.trace_span(w, args)[0] - args.warmup >= 1
+    plain = bench.workload_config(w, bench.parse_args(["--workload", "aq-stress"]), 2, 1)
+    assert "trace_steps" not in plain and plain["arenas_cycled"] == 2
+
+
 def test_host_arena_follows_the_layout_and_the_trace_scales():
     """The reference arm's host-generated arena: the workload's packing,
     zeros outside the units, every unit scaled by the power of two nearest

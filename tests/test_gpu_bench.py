@@ -53,3 +53,14 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
         assert rec["trace_candidates_mean"] >= 0 and 0 <= rec["trace_selected_mean"] <= rec["max_o"]
         assert 0 <= rec["trace_hit_max_o_rate"] <= 1
     assert per["aq-stress"]["candidates_mean"] > per["aq-stress"]["max_o"]   # the contended top-k
+
+
+def test_trace_steps_mode_times_the_trace_window(capsys, cuda_device):
+    """--trace-steps: the timed steps are the workload's own consecutive
+    trace steps, so their candidate counts are the trace's."""
+    bench.main(["--workload", "tiny", "--trace-steps", "--steps", "6", "--warmup", "3", "--no-e2e",
+                "--no-cpu-baseline", "--no-sparsity", "--no-per-workload"])
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    t0, t1 = line["config"]["trace_steps"]
+    assert t1 - t0 + 1 == 6 and t0 >= 4 and line["config"]["arenas_cycled"] == 9
+    assert line["value"] > 0 and line["gpu_launches"] == 6
