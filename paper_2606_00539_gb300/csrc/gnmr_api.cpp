@@ -396,8 +396,8 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         p.static_warmup = c.static_warmup_steps;
         p.static_keep = static_cast<int32_t>(std::min<double>(std::ceil(c.static_fraction * num_rec), num_rec));
         p.num_units = c.num_units;
-        const int32_t warps = static_cast<int32_t>(std::min<int64_t>(plan.num_runs, grid_warps));
-        p.num_warps = warps;
+        const int32_t step_warps = static_cast<int32_t>(std::min<int64_t>(plan.num_runs, grid_warps));
+        p.num_warps = step_warps;
         p.num_runs = plan.num_runs;
         p.window = c.window;
         p.max_o = c.max_o;
@@ -419,9 +419,9 @@ gnmr_status gnmr_create(const gnmr_config *cfg, gnmr_handle **out)
         h->variant = variant;
         h->num_units = c.num_units;
         h->elem_bytes = eb;
-        h->num_warps = warps;
+        h->num_warps = step_warps;
         h->num_runs = plan.num_runs;
-        h->num_ctas = (warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
+        h->num_ctas = (step_warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
         {
             const int64_t warps = (U + 31) / 32;
             const int64_t ctas = (warps + gnmr::kWarpsPerCta - 1) / gnmr::kWarpsPerCta;
