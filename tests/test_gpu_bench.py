@@ -55,11 +55,13 @@ def test_gpu_arm_prints_the_contract_line(capsys, cuda_device):
     assert per["aq-stress"]["candidates_mean"] > per["aq-stress"]["max_o"]   # the contended top-k
 
 
-def test_trace_steps_mode_times_the_trace_window(capsys, cuda_device):
+@pytest.mark.parametrize("graph", [False, True])
+def test_trace_steps_mode_times_the_trace_window(graph, capsys, cuda_device):
     """--trace-steps: the timed steps are the workload's own consecutive
-    trace steps, so their candidate counts are the trace's."""
+    trace steps, so their candidate counts are the trace's (with --graph the
+    untimed first replay's state is restored before the timed one)."""
     bench.main(["--workload", "tiny", "--trace-steps", "--steps", "6", "--warmup", "3", "--no-e2e",
-                "--no-cpu-baseline", "--no-sparsity", "--no-per-workload"])
+                "--no-cpu-baseline", "--no-sparsity", "--no-per-workload"] + (["--graph"] if graph else []))
     line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
     t0, t1 = line["config"]["trace_steps"]
     assert t1 - t0 + 1 == 6 and t0 >= 4 and line["config"]["arenas_cycled"] == 9
