@@ -132,6 +132,44 @@ def test_large_unit_loop_takes_runs_dynamically(cuda_device):
             assert info["num_ctas"] * info["threads_per_cta"] // 32 >= info["num_warps"]
 
 
+def test_two_handles_stepping_concurrently_do_not_interfere(cuda_device):
+    """Two handles of the same large-unit layout (dynamic runs: each handle
+    has its own run counter) stepping on two streams at once, with no host
+    synchronisation between them, give bit-identical outputs to a third
+    handle stepping alone."""
+    import torch
+    w = workloads.make("llama2-1.3b", shrink=2, steps=6)
+    filler = workloads.Filler(w, cuda_device)
+    arenas = []
+    for t in range(w.steps):
+        a = filler.new_arena()
+        filler.fill(a, t)
+        arenas.append(a)
+    torch.cuda.synchronize()
+    mons = [_monitor(w) for _ in range(3)]
+    try:
+        assert mons[0].info()["num_runs"] > mons[0].info()["num_warps"]
+        streams = [torch.cuda.Stream(cuda_device) for _ in range(2)]
+        stats = [m.new_stats() for m in mons]
+        masks = [torch.empty(w.num_units, dtype=torch.uint8, device=cuda_device) for _ in mons]
+        history = [[] for _ in mons]
+        for t in range(w.steps):
+            for k in range(2):                                   # concurrent, no sync between
+                mons[k].step(arenas[t], mask=masks[k], stats=stats[k], stream=streams[k])
+            torch.cuda.synchronize()
+            mons[2].step(arenas[t], mask=masks[2], stats=stats[2])   # alone
+            torch.cuda.synchronize()
+            for k in range(3):
+                history[k].append({n: v.clone() for n, v in stats[k].items()} | {"mask": masks[k].clone()})
+        for t in range(w.steps):
+            for k in range(2):
+                for name, v in history[2][t].items():
+                    assert torch.equal(history[k][t][name], v), (t, k, name)
+    finally:
+        for m in mons:
+            m.close()
+
+
 def test_segments_in_any_order_and_units_without_segments(cuda_device):
     import torch
     rng = np.random.default_rng(21)
