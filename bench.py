@@ -867,7 +867,7 @@ def run_gnmr(args):
                 host = None
 
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:     # the host baseline: N = 1 only
         k = args.cpu_sample_units or w.num_units
         units = np.arange(min(k, w.num_units))
         hi = int(w.offsets[units[-1]] + w.lengths[units[-1]])
